@@ -1,0 +1,210 @@
+"""fp64 CPU oracle of the SOLO shared-readout local loss.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import this module.  It shares no
+code with the CUDA library and never calls it.
+
+What it computes, for every module k and token i (paper, Section 2.2, Eq. 2
+with tau_k = 1 and no bias; Eq. 3; Algorithm 1, the local cross-entropy of
+each module and the terminal cross-entropy that updates W; the head's final
+RMSNorm with element-wise gain, Appendix C "Language" and the ROT/RSHARE
+paragraph of Appendix D):
+
+1. ms_i = (1/d) sum_j h_ij^2,   r_i = 1 / sqrt(ms_i + eps)
+2. xhat_ij = Q(gamma_j h_ij r_i)        Q = bf16 round-to-nearest-even in
+                                         "contract" mode, identity in "exact"
+3. z_iv = sum_j xhat_ij W_vj             (logits through the shared readout)
+4. lse_i = max_v z + ln sum_v exp(z_iv - max_v z)
+   loss_i = lse_i - z_{i,y_i} for kept tokens, 0 otherwise
+   L_k = sum_i loss_i / Nvalid_k (0 when no token is kept)
+5. g_iv = (exp(z_iv - lse_i) - [v = y_i]) / Nvalid_k   (delta_k of Eq. 1,
+   scaled by the mean; zero rows for masked tokens)
+6. dxhat = g W                            (the readout factor W^T delta_k, Eq. 3)
+7. dh_ij = r_i gamma_j dxhat_ij - (r_i^3/d) h_ij sum_l gamma_l dxhat_il h_il
+   (Jacobian of the final RMSNorm)
+8. final module only (Algorithm 1: only the terminal loss updates W):
+   dW_vj = sum_i g_iv xhat_ij,   dgamma_j = sum_i dxhat_ij h_ij r_i
+
+A token is kept when its target lies in [0, V), differs from ignore_index
+and its optional mask byte is non-zero.  A target outside [0, V) that is not
+ignore_index is treated as masked and reported (``bad_target``).
+
+Every step is a plain numpy fp64 expression; the matrix products are the
+only library primitive used.  Rows are independent given Nvalid_k, so
+``module_rows`` may be called on any subset of a module's rows.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+# -- inputs -----------------------------------------------------------------
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) to exact float64 values."""
+    u = np.asarray(bits).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+def round_to_bf16(x: np.ndarray) -> np.ndarray:
+    """Rounds float64 values to the nearest bf16 value, ties to even.
+
+    bf16 keeps 8 significant bits.  With x = m * 2^e, 0.5 <= |m| < 1, the
+    rounded value is rint(256 m) / 256 * 2^e (rint rounds half to even).
+    Rounding happens once, from float64.  bf16 subnormals (|x| < 2^-126) are
+    out of this oracle's range.
+    """
+    m, e = np.frexp(np.asarray(x, dtype=np.float64))
+    return np.ldexp(np.rint(m * 256.0) / 256.0, e)
+
+
+def kept_tokens(targets: np.ndarray, mask, V: int, ignore_index: int):
+    """(kept, bad): kept tokens and targets that are neither valid nor ignore_index."""
+    t = np.asarray(targets)
+    in_range = (t >= 0) & (t < V)
+    bad = (~in_range) & (t != ignore_index)
+    kept = in_range & (t != ignore_index)
+    if mask is not None:
+        kept &= np.asarray(mask) != 0
+    return kept, bad
+
+
+# -- steps 1-2: final RMSNorm with gain --------------------------------------
+
+def rmsnorm_forward(h, gamma, eps, contract=True):
+    d = h.shape[1]
+    ms = np.sum(h * h, axis=1) / d
+    r = 1.0 / np.sqrt(ms + eps)
+    xhat = gamma[None, :] * h * r[:, None]
+    if contract:
+        xhat = round_to_bf16(xhat)
+    return r, xhat
+
+
+# -- steps 3-5: logits, cross-entropy, its gradient ---------------------------
+
+def logits(xhat, W):
+    return xhat @ W.T
+
+
+def log_sum_exp(z):
+    m = np.max(z, axis=1)
+    return m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
+
+
+def token_loss(z, lse, y, kept):
+    rows = np.arange(z.shape[0])
+    yc = np.where(kept, y, 0)
+    return np.where(kept, lse - z[rows, yc], 0.0)
+
+
+def logit_grad(z, lse, y, kept, n_valid):
+    """g = (softmax(z) - onehot(y)) / Nvalid on kept rows, 0 on the others."""
+    g = np.exp(z - lse[:, None])
+    rows = np.nonzero(kept)[0]
+    g[rows, y[rows]] -= 1.0
+    w = np.where(kept, 1.0 / max(n_valid, 1), 0.0)
+    return g * w[:, None]
+
+
+# -- steps 6-8: back through the readout and the norm -------------------------
+
+def input_grad(g, W):
+    return g @ W
+
+
+def rmsnorm_backward(dxhat, h, gamma, r):
+    d = h.shape[1]
+    c = np.sum(gamma[None, :] * dxhat * h, axis=1)
+    return (r[:, None] * gamma[None, :] * dxhat
+            - (r ** 3 / d)[:, None] * h * c[:, None])
+
+
+def readout_grads(g, xhat, dxhat, h, r):
+    """(dW, dgamma) summed over the given rows of the final module."""
+    dW = g.T @ xhat
+    dgamma = np.sum(dxhat * h * r[:, None], axis=0)
+    return dW, dgamma
+
+
+# -- drivers ----------------------------------------------------------------
+
+def module_rows(h, gamma, W, y, kept, n_valid, eps, contract=True):
+    """Every per-token quantity for a set of rows of one module."""
+    r, xhat = rmsnorm_forward(h, gamma, eps, contract)
+    z = logits(xhat, W)
+    lse = log_sum_exp(z)
+    loss = token_loss(z, lse, y, kept)
+    g = logit_grad(z, lse, y, kept, n_valid)
+    dxhat = input_grad(g, W)
+    dh = rmsnorm_backward(dxhat, h, gamma, r)
+    zy = z[np.arange(len(y)), np.where(kept, y, 0)]
+    return dict(r=r, xhat=xhat, z=z, lse=lse, loss=loss, g=g, dxhat=dxhat,
+                dh=dh, zy=zy)
+
+
+def solo_readout_fwd_bwd(hidden, gamma, W, targets, mask=None, eps=1e-6,
+                         ignore_index=-100, contract=True, want_dW=True,
+                         want_dgamma=True):
+    """Full oracle for small problems.
+
+    hidden: sequence of K float64 arrays [N, d]; gamma [d]; W [V, d];
+    targets int [K, N]; mask None or [K, N].  Returns a dict with loss_tok
+    [K, N], loss_mean [K], n_valid [K], dhidden (list of [N, d]), dW [V, d]
+    and dgamma [d] of the final module, bad_target (bool) and per-module
+    intermediates ``rows`` (list of module_rows dicts).
+    """
+    K = len(hidden)
+    V = W.shape[0]
+    out = dict(loss_tok=[], loss_mean=np.zeros(K), n_valid=np.zeros(K, int),
+               dhidden=[], rows=[], bad_target=False)
+    for k in range(K):
+        kept, bad = kept_tokens(targets[k], None if mask is None else mask[k],
+                                V, ignore_index)
+        out["bad_target"] |= bool(bad.any())
+        n_valid = int(kept.sum())
+        res = module_rows(hidden[k], gamma, W, np.asarray(targets[k]), kept,
+                          n_valid, eps, contract)
+        out["loss_tok"].append(res["loss"])
+        out["loss_mean"][k] = res["loss"].sum() / n_valid if n_valid else 0.0
+        out["n_valid"][k] = n_valid
+        out["dhidden"].append(res["dh"])
+        out["rows"].append(res)
+        if k == K - 1:
+            dW, dgamma = readout_grads(res["g"], res["xhat"], res["dxhat"],
+                                       hidden[k], res["r"])
+            if want_dW:
+                out["dW"] = dW
+            if want_dgamma:
+                out["dgamma"] = dgamma
+    out["loss_tok"] = np.stack(out["loss_tok"])
+    return out
+
+
+def final_module_chunked(h_rows_fn, N, gamma, W, y, kept, eps, contract=True,
+                         dW_cols=None, chunk=1024):
+    """Final-module pass over all N rows in chunks, for full-size checks.
+
+    ``h_rows_fn(i0, n)`` returns rows [i0, i0+n) of the module as float64.
+    Returns loss [N], lse [N], dgamma [d], and dW rows ``dW_cols`` (the
+    vocabulary entries v whose dW_v, an [len, d] array, is wanted).
+    """
+    n_valid = int(kept.sum())
+    d = W.shape[1]
+    loss = np.zeros(N)
+    lse = np.zeros(N)
+    dgamma = np.zeros(d)
+    cols = None if dW_cols is None else np.asarray(dW_cols)
+    dW_part = None if cols is None else np.zeros((len(cols), d))
+    for i0 in range(0, N, chunk):
+        n = min(chunk, N - i0)
+        h = h_rows_fn(i0, n)
+        res = module_rows(h, gamma, W, y[i0:i0 + n], kept[i0:i0 + n], n_valid,
+                          eps, contract)
+        loss[i0:i0 + n] = res["loss"]
+        lse[i0:i0 + n] = res["lse"]
+        dgamma += np.sum(res["dxhat"] * h * res["r"][:, None], axis=0)
+        if cols is not None:
+            dW_part += res["g"][:, cols].T @ res["xhat"]
+    return dict(loss=loss, lse=lse, dgamma=dgamma, dW_rows=dW_part,
+                n_valid=n_valid)

@@ -1,0 +1,286 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle.
+
+Each ``pin_*`` function raises AssertionError when the oracle disagrees with
+a closed form, an invariant, brute force, finite differences or an
+independent PyTorch fp64 composition.  ``test_oracle_pins.py`` runs them on
+the oracle as written, and ``test_oracle_mutations.py`` runs them on copies
+of the oracle with a planted mistake to show that each mistake is caught.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+from paper_2609_35440_gb300 import synth
+from paper_2609_35440_gb300.workloads import Workload
+
+
+def problem(K=2, N=6, d=8, V=16, seed=11, mask_frac=0.0, row_scale=False,
+            heavy=0.0, targets="uniform", keep_mask=None, orc=None):
+    """A small fp64 problem decoded from the seeded bf16 generator."""
+    wl = Workload("pin", K=K, N=N, d=d, V=V, seed=seed, mask_frac=mask_frac,
+                  row_scale=row_scale, heavy_frac=heavy, targets=targets)
+    inp = synth.generate(wl)
+    dec = orc.bf16_bits_to_f64
+    hidden = [dec(inp.hidden[k]) for k in range(K)]
+    return dict(hidden=hidden, gamma=dec(inp.gamma), W=dec(inp.W),
+                targets=inp.targets.astype(np.int64), mask=keep_mask,
+                eps=wl.eps, V=V, d=d, K=K, N=N)
+
+
+def run(orc, p, contract=False, **kw):
+    args = dict(hidden=p["hidden"], gamma=p["gamma"], W=p["W"],
+                targets=p["targets"], mask=p["mask"], eps=p["eps"],
+                contract=contract)
+    args.update(kw)
+    return orc.solo_readout_fwd_bwd(**args)
+
+
+def rel(a, b):
+    a, b = np.asarray(a, float), np.asarray(b, float)
+    den = np.max(np.abs(b))
+    return float(np.max(np.abs(a - b)) / (den if den > 0 else 1.0))
+
+
+# -- bf16 rounding ------------------------------------------------------------
+
+def pin_bf16_rounding(orc):
+    q = orc.round_to_bf16
+    cases = [
+        (1.0, 1.0),
+        (1.0 + 2.0 ** -8, 1.0),                       # tie -> even (down)
+        (1.0 + 3 * 2.0 ** -8, 1.0 + 2.0 ** -6),      # tie -> even (up)
+        (1.0 + 2.0 ** -8 + 2.0 ** -40, 1.0 + 2.0 ** -7),  # above tie: up
+        (-(1.0 + 2.0 ** -8), -1.0),
+        (3.0 * 2.0 ** 20 + 2.0 ** 13, 3.0 * 2.0 ** 20),  # 8 significant bits
+        (255.5, 256.0),                               # tie at 9 bits -> even
+        (254.5, 254.0),
+        (0.0, 0.0),
+        (1.0 / 3.0, 0.333984375),
+    ]
+    for x, want in cases:
+        got = float(q(np.array([x]))[0])
+        assert got == want, (x, got, want)
+
+
+# -- loss ---------------------------------------------------------------------
+
+def pin_zero_readout(orc):
+    """W = 0: loss = ln V exactly, dH = dgamma = 0, dW in closed form."""
+    p = problem(K=2, N=7, d=8, V=24, seed=3, mask_frac=0.3, orc=orc)
+    p["W"] = np.zeros_like(p["W"])
+    for contract in (False, True):
+        out = run(orc, p, contract=contract)
+        K, V = p["K"], p["V"]
+        kept, _ = orc.kept_tokens(p["targets"][K - 1], None, V, -100)
+        for k in range(K):
+            kk, _ = orc.kept_tokens(p["targets"][k], None, V, -100)
+            np.testing.assert_allclose(out["loss_tok"][k][kk], math.log(V), rtol=0, atol=1e-13)
+            assert np.all(out["loss_tok"][k][~kk] == 0.0)
+            np.testing.assert_allclose(out["loss_mean"][k], math.log(V), rtol=0, atol=1e-13)
+            assert np.all(out["dhidden"][k] == 0.0)
+        assert np.all(out["dgamma"] == 0.0)
+        # closed form: dW = (1/Nvalid) sum_i (1/V - e_{y_i}) xhat_i^T
+        h = p["hidden"][K - 1]
+        ms = np.array([sum(v * v for v in row) / p["d"] for row in h])
+        xhat = p["gamma"][None, :] * h / np.sqrt(ms + p["eps"])[:, None]
+        if contract:
+            xhat = orc.round_to_bf16(xhat)
+        nv = kept.sum()
+        want = np.zeros((V, p["d"]))
+        for i in np.nonzero(kept)[0]:
+            want += xhat[i][None, :] / V
+            want[p["targets"][K - 1][i]] -= xhat[i]
+        want /= nv
+        np.testing.assert_allclose(out["dW"], want, rtol=1e-12, atol=1e-15)
+
+
+def pin_brute_force_ce(orc):
+    """Per-token CE from explicit loops, no max shift, small logits."""
+    p = problem(K=1, N=5, d=6, V=12, seed=5, orc=orc)
+    p["W"] = p["W"] * 10.0          # logits of order one
+    out = run(orc, p, contract=False)
+    h, g, W = p["hidden"][0], p["gamma"], p["W"]
+    d, V = p["d"], p["V"]
+    for i in range(p["N"]):
+        ms = sum(h[i][j] ** 2 for j in range(d)) / d
+        r = 1.0 / math.sqrt(ms + p["eps"])
+        x = [g[j] * h[i][j] * r for j in range(d)]
+        z = [sum(x[j] * W[v][j] for j in range(d)) for v in range(V)]
+        want = math.log(sum(math.exp(zv) for zv in z)) - z[p["targets"][0][i]]
+        assert abs(out["loss_tok"][0][i] - want) < 1e-12, (i, out["loss_tok"][0][i], want)
+
+
+# -- gradients ----------------------------------------------------------------
+
+def _loss_k(orc, p, k, **over):
+    q = dict(p)
+    q.update(over)
+    return run(orc, q, contract=False)["loss_mean"][k]
+
+
+def pin_finite_differences(orc):
+    """Central differences of the module losses (exact mode, fp64)."""
+    p = problem(K=2, N=4, d=8, V=16, seed=7, mask_frac=0.25, row_scale=True, orc=orc)
+    p["W"] = p["W"] * 20.0
+    out = run(orc, p, contract=False)
+    K, step = p["K"], 1e-6
+    for k in range(K):
+        num = np.zeros_like(p["hidden"][k])
+        for idx in np.ndindex(*num.shape):
+            hp = [h.copy() for h in p["hidden"]]
+            hm = [h.copy() for h in p["hidden"]]
+            hp[k][idx] += step
+            hm[k][idx] -= step
+            num[idx] = (_loss_k(orc, p, k, hidden=hp) - _loss_k(orc, p, k, hidden=hm)) / (2 * step)
+        assert rel(out["dhidden"][k], num) < 1e-7, ("dH", k, rel(out["dhidden"][k], num))
+    numW = np.zeros_like(p["W"])
+    for idx in np.ndindex(*numW.shape):
+        Wp, Wm = p["W"].copy(), p["W"].copy()
+        Wp[idx] += step
+        Wm[idx] -= step
+        numW[idx] = (_loss_k(orc, p, K - 1, W=Wp) - _loss_k(orc, p, K - 1, W=Wm)) / (2 * step)
+    assert rel(out["dW"], numW) < 1e-7, ("dW", rel(out["dW"], numW))
+    numg = np.zeros_like(p["gamma"])
+    for j in range(len(numg)):
+        gp, gm = p["gamma"].copy(), p["gamma"].copy()
+        gp[j] += step
+        gm[j] -= step
+        numg[j] = (_loss_k(orc, p, K - 1, gamma=gp) - _loss_k(orc, p, K - 1, gamma=gm)) / (2 * step)
+    assert rel(out["dgamma"], numg) < 1e-7, ("dgamma", rel(out["dgamma"], numg))
+
+
+def pin_softmax_rows_sum_to_zero(orc):
+    """Rows of (softmax - onehot) sum to zero; adding a common row to W changes nothing."""
+    p = problem(K=2, N=9, d=16, V=40, seed=9, mask_frac=0.2, orc=orc)
+    p["W"] = p["W"] * 30.0
+    out = run(orc, p, contract=False)
+    for res in out["rows"]:
+        assert np.max(np.abs(res["g"].sum(axis=1))) < 1e-15
+    c = np.linspace(-0.5, 0.7, p["d"])
+    out2 = run(orc, dict(p, W=p["W"] + c[None, :]), contract=False)
+    for k in range(p["K"]):
+        np.testing.assert_allclose(out2["loss_tok"][k], out["loss_tok"][k], rtol=0, atol=1e-11)
+        assert rel(out2["dhidden"][k], out["dhidden"][k]) < 1e-9
+    # each column of dW sums to zero over the vocabulary
+    colsum = out["dW"].sum(axis=0)
+    assert np.max(np.abs(colsum)) < 1e-14 * max(1.0, np.max(np.abs(out["dW"])))
+
+
+def pin_scale_invariance(orc):
+    """With eps = 0 the loss is degree-0 homogeneous in h: dH(a h) = dH(h)/a and <dh_i, h_i> = 0."""
+    p = problem(K=1, N=6, d=16, V=32, seed=13, orc=orc)
+    p["W"] = p["W"] * 10.0
+    p["eps"] = 0.0
+    out = run(orc, p, contract=False)
+    a = 3.7
+    out2 = run(orc, dict(p, hidden=[h * a for h in p["hidden"]]), contract=False)
+    np.testing.assert_allclose(out2["loss_tok"], out["loss_tok"], rtol=1e-12, atol=1e-13)
+    assert rel(out2["dhidden"][0] * a, out["dhidden"][0]) < 1e-11
+    dh, h = out["dhidden"][0], p["hidden"][0]
+    euler = np.abs(np.sum(dh * h, axis=1)) / (np.linalg.norm(dh, axis=1) * np.linalg.norm(h, axis=1))
+    assert np.max(euler) < 1e-12
+
+
+def pin_masking(orc):
+    """Masked tokens: zero loss and an exactly-zero dH row; out of range = masked + flagged."""
+    p = problem(K=2, N=8, d=8, V=16, seed=15, orc=orc)
+    keep = np.ones((2, 8), dtype=np.uint8)
+    keep[0, [1, 5]] = 0
+    p["mask"] = keep
+    tg = p["targets"].copy()
+    tg[1, 2] = -100
+    tg[1, 6] = 16            # out of range -> masked and flagged
+    p["targets"] = tg
+    out = run(orc, p, contract=True)
+    assert out["bad_target"]
+    for k, rows in ((0, [1, 5]), (1, [2, 6])):
+        assert np.all(out["loss_tok"][k][rows] == 0.0)
+        assert np.all(out["dhidden"][k][rows] == 0.0)
+        assert out["n_valid"][k] == 6
+        kept = np.ones(8, bool)
+        kept[rows] = False
+        np.testing.assert_allclose(out["loss_mean"][k], out["loss_tok"][k][kept].mean(), rtol=1e-14)
+    # a module with no kept token: zero loss, zero gradients
+    p["targets"] = np.full_like(tg, -100)
+    out = run(orc, p, contract=True)
+    assert np.all(out["loss_mean"] == 0.0) and not out["bad_target"]
+    assert all(np.all(dh == 0.0) for dh in out["dhidden"])
+    assert np.all(out["dW"] == 0.0) and np.all(out["dgamma"] == 0.0)
+
+
+def pin_dgamma_identity(orc):
+    """sum_j gamma_j dgamma_j = sum_i <dxhat_i, xhat_i> (exact mode)."""
+    p = problem(K=2, N=10, d=16, V=32, seed=17, row_scale=True, orc=orc)
+    p["W"] = p["W"] * 10.0
+    out = run(orc, p, contract=False)
+    res = out["rows"][-1]
+    lhs = float(np.dot(p["gamma"], out["dgamma"]))
+    rhs = float(np.sum(res["dxhat"] * res["xhat"]))
+    assert abs(lhs - rhs) <= 1e-12 * max(1.0, abs(rhs)), (lhs, rhs)
+
+
+def pin_torch_fp64(orc):
+    """Independent composition of library routines: F.rms_norm, matmul, F.cross_entropy, autograd."""
+    import torch
+    import torch.nn.functional as F
+    p = problem(K=3, N=11, d=24, V=50, seed=19, mask_frac=0.2, row_scale=True,
+                heavy=0.1, orc=orc)
+    p["W"] = p["W"] * 5.0
+    out = run(orc, p, contract=False)
+    W = torch.tensor(p["W"], dtype=torch.float64, requires_grad=True)
+    g = torch.tensor(p["gamma"], dtype=torch.float64, requires_grad=True)
+    for k in range(p["K"]):
+        h = torch.tensor(p["hidden"][k], dtype=torch.float64, requires_grad=True)
+        y = torch.tensor(p["targets"][k], dtype=torch.int64)
+        x = F.rms_norm(h, (p["d"],), weight=g, eps=p["eps"])
+        loss = F.cross_entropy(x @ W.T, y, ignore_index=-100)
+        W.grad = None
+        g.grad = None
+        loss.backward()
+        assert abs(loss.item() - out["loss_mean"][k]) < 1e-12
+        assert rel(out["dhidden"][k], h.grad.numpy()) < 1e-11
+        if k == p["K"] - 1:
+            assert rel(out["dW"], W.grad.numpy()) < 1e-11
+            assert rel(out["dgamma"], g.grad.numpy()) < 1e-11
+
+
+def pin_row_subsets(orc):
+    """module_rows on a subset and the chunked final-module pass agree with the full oracle."""
+    p = problem(K=2, N=37, d=16, V=64, seed=21, mask_frac=0.2, orc=orc)
+    out = run(orc, p, contract=True)
+    k = 1
+    kept, _ = orc.kept_tokens(p["targets"][k], None, p["V"], -100)
+    rows = np.array([0, 5, 17, 36])
+    sub = orc.module_rows(p["hidden"][k][rows], p["gamma"], p["W"], p["targets"][k][rows],
+                          kept[rows], int(kept.sum()), p["eps"], True)
+    np.testing.assert_allclose(sub["loss"], out["loss_tok"][k][rows], rtol=1e-15, atol=0)
+    np.testing.assert_allclose(sub["dh"], out["dhidden"][k][rows], rtol=1e-15, atol=0)
+    cols = np.array([0, 3, 63])
+    ch = orc.final_module_chunked(lambda i0, n: p["hidden"][k][i0:i0 + n], p["N"], p["gamma"],
+                                  p["W"], p["targets"][k], kept, p["eps"], True, dW_cols=cols,
+                                  chunk=8)
+    np.testing.assert_allclose(ch["loss"], out["loss_tok"][k], rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(ch["dgamma"], out["dgamma"], rtol=1e-12, atol=1e-18)
+    np.testing.assert_allclose(ch["dW_rows"], out["dW"][cols], rtol=1e-12, atol=1e-18)
+
+
+def pin_init_statistics(orc):
+    """At init, lse_i = ln V + sigma_i^2/2 to first order with sigma_i^2 = |xhat_i|^2 E[W^2],
+    and the mean loss differs from the mean lse by the mean target logit, which is
+    zero-mean with spread sigma/sqrt(N)."""
+    p = problem(K=1, N=256, d=256, V=2048, seed=23, orc=orc)
+    out = run(orc, p, contract=True)
+    res = out["rows"][0]
+    s2 = np.sum(res["xhat"] ** 2, axis=1) * np.mean(p["W"] ** 2)
+    want = math.log(p["V"]) + s2 / 2.0
+    assert np.max(np.abs(res["lse"] - want)) < 0.2 * np.max(s2) ** 2 + 0.02, np.max(np.abs(res["lse"] - want))
+    assert abs(np.mean(res["lse"]) - np.mean(want)) < 0.01
+    spread = math.sqrt(float(np.mean(s2)) / p["N"])
+    assert abs(out["loss_mean"][0] - np.mean(res["lse"])) < 4 * spread
+
+
+PINS = [pin_bf16_rounding, pin_zero_readout, pin_brute_force_ce, pin_finite_differences,
+        pin_softmax_rows_sum_to_zero, pin_scale_invariance, pin_masking, pin_dgamma_identity,
+        pin_torch_fp64, pin_row_subsets, pin_init_statistics]
