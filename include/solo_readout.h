@@ -1,0 +1,181 @@
+/*
+ * solo_readout.h -- C ABI of the SOLO shared-readout local loss on one GB300.
+ *
+ * SOLO (Shared-Output LOcal learning) splits a network into K
+ * gradient-isolated modules.  Every module k predicts the next token through
+ * a read-only copy of the terminal readout (paper, Section 2.2, Eq. 2 with
+ * temperature tau_k = 1 and no bias):
+ *
+ *     xhat_i  = RMSNorm_gamma(h_i)          final RMSNorm with element-wise gain
+ *     z_i     = W xhat_i                     W: [V, d], the terminal readout
+ *     loss_i  = logsumexp(z_i) - z_{i, y_i}  cross-entropy against next token
+ *     L_k     = mean of loss_i over the kept tokens of module k
+ *
+ * and receives only its own gradient back through the same readout (Eq. 3):
+ * dL_k/dh_k = J_norm^T W^T (softmax(z) - onehot(y)) / Nvalid_k.  No gradient
+ * ever reaches the copy of W; only the final module's loss updates W and
+ * gamma (Algorithm 1, the terminal cross-entropy and the Step that follows
+ * it), so dW and dgamma are produced for module K-1 (0-based) alone.
+ *
+ * Conventions for every entry point:
+ *  - Pointers are DEVICE pointers unless the comment says "host".  The caller
+ *    owns all memory; the library allocates nothing and keeps no state
+ *    between calls besides per-device kernel attributes set on first use.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream).  Errors the host can detect are returned before any
+ *    work is enqueued; conditions found on the device set bits of a flag
+ *    word in the workspace, read back with solo_readout_get_flags.
+ *  - bf16 tensors are passed as their 16-bit patterns (solo_bf16_t).
+ *  - Row-major layouts; every tensor pointer must be 16-byte aligned.
+ *  - Calls using distinct workspaces may run concurrently on different
+ *    streams.  W and gamma must not be written while a call that reads them
+ *    is in flight (they are the read-only copy of Algorithm 1).
+ *  - Requires a compute capability 10.3 device (GB300, sm_103a).
+ */
+#ifndef SOLO_READOUT_H
+#define SOLO_READOUT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t solo_bf16_t;          /* bf16 bit pattern */
+typedef struct CUstream_st* solo_stream_t; /* same type as cudaStream_t */
+typedef int32_t solo_status_t;
+
+enum {
+  SOLO_OK = 0,
+  SOLO_ERR_INVALID_ARG = -1,         /* NULL required pointer, K/N/d/V out of range */
+  SOLO_ERR_UNSUPPORTED_SHAPE = -2,   /* d not a multiple of 8 */
+  SOLO_ERR_WORKSPACE_TOO_SMALL = -3, /* workspace_bytes below the query result */
+  SOLO_ERR_CUDA = -4,                /* a CUDA runtime call failed */
+  SOLO_ERR_NOT_SM103 = -5,           /* current device is not compute capability 10.3 */
+  SOLO_ERR_MISALIGNED = -6           /* a tensor pointer is not 16-byte aligned */
+};
+
+/* Device-detected conditions, OR-ed into the workspace flag word. */
+enum {
+  SOLO_FLAG_BAD_TARGET = 1u, /* a target outside [0, V) that is not ignore_index;
+                                the token is treated as masked */
+  SOLO_FLAG_TIMEOUT = 2u     /* a pipeline wait exceeded its bound (about 2 s);
+                                the kernel stopped early and outputs are invalid */
+};
+
+/* Maximum number of modules per call. */
+#define SOLO_MAX_MODULES 16
+
+/* Stages of one call, for solo_readout_fwd_bwd_events. */
+enum {
+  SOLO_STAGE_RMSNORM = 0,   /* r_i and xhat = bf16(gamma * h * r)           */
+  SOLO_STAGE_LOGITS = 1,    /* tensor-core X W^T, per-tile max/sum, exps    */
+  SOLO_STAGE_LSE = 2,       /* logsumexp, token loss, module means          */
+  SOLO_STAGE_GRAD = 3,      /* dL/dz = (softmax - onehot) / Nvalid, bf16    */
+  SOLO_STAGE_DXHAT = 4,     /* tensor-core dXhat = G W                      */
+  SOLO_STAGE_NORM_BWD = 5,  /* dH through the RMSNorm Jacobian, dgamma parts */
+  SOLO_STAGE_DW = 6,        /* tensor-core dW = G^T Xhat, final module      */
+  SOLO_STAGE_DGAMMA = 7,    /* dgamma reduction, final module               */
+  SOLO_NUM_STAGES = 8
+};
+
+typedef struct {
+  int32_t K;            /* modules, 1 .. SOLO_MAX_MODULES                    */
+  int64_t N;            /* tokens per module, >= 1                           */
+  int32_t d;            /* width, >= 8 and a multiple of 8                   */
+  int32_t V;            /* vocabulary size, >= 1                             */
+  float eps;            /* RMSNorm epsilon, inside the square root (>= 0)    */
+  int32_t ignore_index; /* target value of a masked token (e.g. -100)        */
+} solo_dims_t;
+
+/*
+ * Bytes of device workspace one call with these dims needs (host-only; no
+ * CUDA call).  The workspace holds the normalised inputs, the bf16
+ * exponentials/gradient of the logits ([K*N, V]), per-token statistics and
+ * the flag word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims
+ * out of range, SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0.
+ */
+solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
+
+/*
+ * One forward + backward of the shared-readout local loss for all K modules
+ * (Eq. 2-3; Algorithm 1, the local cross-entropy of every module and the
+ * terminal cross-entropy of the last).  All K modules run as one row space
+ * of K*N tokens against one resident W.
+ *
+ *  hidden     host array [K] of device pointers, each bf16 [N, d]: h_k, the
+ *             head output of module k before its final RMSNorm.
+ *  gamma      bf16 [d]: the final RMSNorm gain.
+ *  W          bf16 [V, d]: the readout; W-bar == W for this call. Never written.
+ *  targets    int32 [K, N]: next-token ids, already shifted; ignore_index
+ *             marks masked tokens; anything else outside [0, V) is treated
+ *             as masked and sets SOLO_FLAG_BAD_TARGET.
+ *  mask       uint8 [K, N] or NULL: 0 masks the token (ANDed with the above).
+ *  loss_tok   fp32 [K, N] or NULL: per-token cross-entropy, 0 when masked.
+ *  loss_mean  fp32 [K]: L_k, mean over kept tokens (0 when none is kept).
+ *  dhidden    host array [K] of device pointers, each bf16 [N, d]:
+ *             dL_k/dh_k.  Rows of masked tokens are exactly 0.
+ *  dW         fp32 [V, d] or NULL: dL_{K-1}/dW (final module), overwritten.
+ *  dgamma     fp32 [d] or NULL: dL_{K-1}/dgamma (final module), overwritten.
+ *  workspace  device buffer of at least solo_readout_workspace_bytes bytes,
+ *             16-byte aligned; its contents on entry do not matter.
+ *
+ * Output buffers may not alias inputs or each other.  Returns SOLO_OK once
+ * the work is enqueued.
+ */
+solo_status_t solo_readout_fwd_bwd(const solo_dims_t* dims,
+                                   const solo_bf16_t* const* hidden,
+                                   const solo_bf16_t* gamma,
+                                   const solo_bf16_t* W,
+                                   const int32_t* targets,
+                                   const uint8_t* mask,
+                                   float* loss_tok,
+                                   float* loss_mean,
+                                   solo_bf16_t* const* dhidden,
+                                   float* dW,
+                                   float* dgamma,
+                                   void* workspace, size_t workspace_bytes,
+                                   solo_stream_t stream);
+
+/*
+ * Same as solo_readout_fwd_bwd, and records events[s] on `stream` right
+ * before stage s is enqueued and events[SOLO_NUM_STAGES] after the last, so
+ * that consecutive events bracket one stage (skipped stages have zero
+ * length).  `events` is a host array of n_events cudaEvent_t handles created
+ * by the caller; n_events must be SOLO_NUM_STAGES + 1.
+ */
+solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
+                                          const solo_bf16_t* const* hidden,
+                                          const solo_bf16_t* gamma,
+                                          const solo_bf16_t* W,
+                                          const int32_t* targets,
+                                          const uint8_t* mask,
+                                          float* loss_tok,
+                                          float* loss_mean,
+                                          solo_bf16_t* const* dhidden,
+                                          float* dW,
+                                          float* dgamma,
+                                          void* workspace, size_t workspace_bytes,
+                                          solo_stream_t stream,
+                                          void* const* events, int32_t n_events);
+
+/*
+ * Waits for `stream`, then copies the flag word of the last call that used
+ * `workspace` into *flags (host).  The word is cleared at the start of
+ * every call.
+ */
+solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream,
+                                     uint32_t* flags);
+
+/* Static description of a status code (never NULL). */
+const char* solo_readout_strerror(solo_status_t status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t solo_readout_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SOLO_READOUT_H */

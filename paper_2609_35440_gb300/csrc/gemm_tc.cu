@@ -1,0 +1,383 @@
+// Persistent tcgen05 GEMM for sm_103a with three fused epilogues.
+//
+// One CTA per SM loops over 128 x 256 output tiles.  Warp 0 streams 64-wide
+// reduction blocks of A and B into a 4-stage shared-memory ring with TMA
+// (128-byte swizzle), warp 1 issues tcgen05.mma (M=128, N=256, K=16, bf16 in,
+// fp32 accumulate) into one of two TMEM accumulators of 256 columns, and
+// warps 2-5 drain the other accumulator (each warp owns 32 TMEM lanes = 32
+// rows of the tile) while the next tile is being multiplied.
+//
+// Epilogues:
+//  kLogits  Z = Xhat W^T.  Per row and tile: m = max_v z, s = sum_v exp(z - m),
+//           the target logit when the target falls in the tile, and the bf16
+//           values exp(z - m) written to a [rows, V] buffer with TMA stores.
+//           These feed the log-sum-exp of the cross-entropy (Eq. 2 and the
+//           local loss of Algorithm 1) and, rescaled, its gradient, so the
+//           logits are never written and never recomputed.
+//  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3; fp32 out.
+//  kDW      dW = G^T Xhat over the final module's tokens; fp32 out.
+//
+// Every wait is bounded (ptx.cuh); on a timeout all roles unwind, in-flight
+// copies and MMAs are drained, TMEM is freed and SOLO_FLAG_TIMEOUT is set.
+#include "internal.h"
+#include "ptx.cuh"
+#include "../../include/solo_readout.h"
+
+namespace solo {
+namespace {
+
+constexpr int kABytes = kBM * kBK * 2;              // 16 KB
+constexpr int kBBytes = kBN * kBK * 2;              // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kEpiBufBytes = 32 * 128;              // 32 rows x 128 B
+constexpr int kEpiWarps = 4;
+constexpr int kTmemCols = 2 * kBN;                  // two accumulators
+constexpr int kSmemA = 0;
+constexpr int kSmemB = kStages * kABytes;
+constexpr int kSmemEpi = kSmemB + kStages * kBBytes;
+constexpr int kSmemBar = kSmemEpi + kEpiWarps * 2 * kEpiBufBytes;
+constexpr int kNumBars = 2 * kStages + 2 + 2 + 1;
+constexpr int kSmemMisc = kSmemBar + kNumBars * 8;
+constexpr int kSmemTotal = kSmemMisc + 16 + 1024;   // + alignment slack
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, int& nb) {
+  const int per_group = a.group_m * a.n_blocks;
+  const int g = t / per_group;
+  const int first_m = g * a.group_m;
+  const int gm = min(a.m_blocks - first_m, a.group_m);
+  const int r = t - g * per_group;
+  mb = first_m + r % gm;
+  nb = r / gm;
+}
+
+// Waits without looking at the abort flag, bounded in time: used to drain
+// copies and MMAs that were already issued when a role gave up.
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const uint32_t a = smem_u32(bar);
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(a, parity)) {
+    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmD, const GemmArgs args) {
+  constexpr bool kAmn = (MODE == kDW);
+  constexpr bool kBmn = (MODE != kLogits);
+  constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN, kAmn, kBmn);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kSmemBar);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kStages;
+  uint64_t* tfull = bars + 2 * kStages;
+  uint64_t* tempty = bars + 2 * kStages + 2;
+  uint64_t* drain = bars + 2 * kStages + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kSmemMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kSmemMisc + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbarrier_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmD);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      uint32_t issued = 0, last_phase = 0;   // per-stage bits for draining
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < args.num_tiles; t += gridDim.x) {
+        int mb, nb;
+        tile_coords(t, args, mb, nb);
+        const int m0 = mb * kBM, n0 = nb * kBN;
+        for (int kb = 0; kb < args.k_blocks; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sA = smem + kSmemA + stage * kABytes;
+          uint8_t* sB = smem + kSmemB + stage * kBBytes;
+          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          const int kr = args.k_row0 + kb * kBK;
+          if constexpr (!kAmn) {
+            tma_load_2d(sA, &tmA, &full[stage], kb * kBK, m0);
+          } else {
+#pragma unroll
+            for (int c = 0; c < kBM / 64; ++c)
+              tma_load_2d(sA + c * 8192, &tmA, &full[stage], m0 + 64 * c, kr);
+          }
+          if constexpr (!kBmn) {
+            tma_load_2d(sB, &tmB, &full[stage], kb * kBK, n0);
+          } else {
+#pragma unroll
+            for (int c = 0; c < kBN / 64; ++c)
+              tma_load_2d(sB + c * 8192, &tmB, &full[stage], n0 + 64 * c, kr);
+          }
+          issued |= 1u << stage;
+          last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (ok) {
+        // Tail: wait until the MMA warp has released every stage, so that no
+        // tcgen05.commit arrival is still pending when the CTA exits.
+        for (int i = 0; ok && i < kStages; ++i) {
+          ok = mbar_wait(&empty[stage], phase ^ 1, abort_flag);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (!ok) {
+        atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
+        for (int s = 0; s < kStages; ++s)
+          if (issued & (1u << s)) mbar_drain(&full[s], (last_phase >> s) & 1u);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      int local = 0;
+      bool ok = true;
+      const uint32_t a_base = smem_u32(smem + kSmemA);
+      const uint32_t b_base = smem_u32(smem + kSmemB);
+      for (int t = blockIdx.x; ok && t < args.num_tiles; t += gridDim.x, ++local) {
+        const uint32_t acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * kBN;
+        for (int kb = 0; kb < args.k_blocks; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = a_base + stage * kABytes;
+          const uint32_t sb = b_base + stage * kBBytes;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            const uint64_t ad = kAmn ? smem_desc_sw128(sa + k * 2048, 8192, 1024)
+                                     : smem_desc_sw128(sa + k * 32, 16, 1024);
+            const uint64_t bd = kBmn ? smem_desc_sw128(sb + k * 2048, 8192, 1024)
+                                     : smem_desc_sw128(sb + k * 32, 16, 1024);
+            mma_bf16(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          mma_commit(&empty[stage]);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit(&tfull[acc]);
+      }
+      if (!ok) {
+        atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
+        mma_commit(drain);
+        mbar_drain(drain, 0);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;                  // TMEM lane quadrant = row block of 32
+    const int ew = warp - 2;                 // staging buffer owner
+    uint8_t* ebuf = smem + kSmemEpi + ew * 2 * kEpiBufBytes;
+    int buf = 0;
+    int local = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < args.num_tiles; t += gridDim.x, ++local) {
+      int mb, nb;
+      tile_coords(t, args, mb, nb);
+      const int m0 = mb * kBM, n0 = nb * kBN;
+      const uint32_t acc = local & 1;
+      const uint32_t acc_phase = (local >> 1) & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + acc * kBN;
+      const int row = m0 + 32 * q + lane;
+      const int ncols = min(kBN, args.N - n0);    // valid columns, warp-uniform
+
+      if constexpr (MODE == kLogits) {
+        const bool row_ok = row < args.M;
+        const int y = row_ok ? args.targets[row] : -1;
+        const int yrel = y - n0;
+        const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
+        float mx = -INFINITY, zyv = 0.f;
+        for (int c = 0; c < kBN / 32; ++c) {
+          if (c * 32 >= ncols) break;
+          float v[32];
+          tmem_ld32(tbase + c * 32, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (c * 32 + j < ncols) mx = fmaxf(mx, v[j]);
+          if (has_y && (yrel >> 5) == c) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j == (yrel & 31)) zyv = v[j];
+          }
+        }
+        const float mlog = mx * kLog2e;
+        float ssum = 0.f;
+        for (int cp = 0; cp < kBN / 64; ++cp) {
+          if (cp * 64 >= ncols) break;
+          if (lane == 0) bulk_wait_group_read<1>();
+          __syncwarp();
+          const uint32_t srow = smem_u32(ebuf + buf * kEpiBufBytes) + lane * 128;
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int c = 2 * cp + half;
+            float v[32];
+            if (c * 32 < ncols) {
+              tmem_ld32(tbase + c * 32, v);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) v[j] = -INFINITY;
+            }
+            uint32_t p[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int col = c * 32 + 2 * j;
+              const float e0 = col < ncols ? ex2_approx(fmaf(v[2 * j], kLog2e, -mlog)) : 0.f;
+              const float e1 = col + 1 < ncols ? ex2_approx(fmaf(v[2 * j + 1], kLog2e, -mlog)) : 0.f;
+              ssum += e0 + e1;
+              p[j] = pack_bf16x2(e0, e1);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const uint32_t chunk = static_cast<uint32_t>(half * 4 + u) ^ (lane & 7);
+              st_shared_v4(srow + (chunk << 4), p[4 * u], p[4 * u + 1], p[4 * u + 2],
+                           p[4 * u + 3]);
+            }
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + cp * 64, m0 + 32 * q);
+            bulk_commit_group();
+          }
+          buf ^= 1;
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+        if (row_ok) args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
+        if (has_y) args.zy[row] = zyv;
+      } else {
+        for (int c = 0; c < kBN / 32; ++c) {
+          if (c * 32 >= ncols) break;
+          float v[32];
+          tmem_ld32(tbase + c * 32, v);
+          if (lane == 0) bulk_wait_group_read<1>();
+          __syncwarp();
+          const uint32_t srow = smem_u32(ebuf + buf * kEpiBufBytes) + lane * 128;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const uint32_t chunk = static_cast<uint32_t>(u) ^ (lane & 7);
+            st_shared_v4(srow + (chunk << 4), __float_as_uint(v[4 * u]),
+                         __float_as_uint(v[4 * u + 1]), __float_as_uint(v[4 * u + 2]),
+                         __float_as_uint(v[4 * u + 3]));
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
+            bulk_commit_group();
+          }
+          buf ^= 1;
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[acc]);
+      }
+    }
+    if (!ok && lane == 0) atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
+    if (lane == 0) bulk_wait_group<0>();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+template <int MODE>
+cudaError_t set_smem_attr() {
+  return cudaFuncSetAttribute(gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kSmemTotal);
+}
+
+}  // namespace
+
+size_t gemm_smem_bytes() { return kSmemTotal; }
+
+cudaError_t gemm_prepare(int /*device*/) {
+  cudaError_t e = set_smem_attr<kLogits>();
+  if (e == cudaSuccess) e = set_smem_attr<kDxhat>();
+  if (e == cudaSuccess) e = set_smem_attr<kDW>();
+  return e;
+}
+
+cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
+                        const CUtensorMap& d, const GemmArgs& args, int grid,
+                        cudaStream_t stream) {
+  if (args.num_tiles <= 0) return cudaSuccess;
+  switch (mode) {
+    case kLogits:
+      gemm_kernel<kLogits><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      break;
+    case kDxhat:
+      gemm_kernel<kDxhat><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      break;
+    case kDW:
+      gemm_kernel<kDW><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      break;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace solo

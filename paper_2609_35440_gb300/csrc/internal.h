@@ -1,0 +1,93 @@
+// Declarations shared by the translation units of libsolo_readout.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace solo {
+
+// Tensor-core tile: 128 rows x 256 columns per CTA, reduction in blocks of 64.
+constexpr int kBM = 128;
+constexpr int kBN = 256;
+constexpr int kBK = 64;
+constexpr int kStages = 4;
+constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
+
+// The three products of one call.
+enum GemmMode : int {
+  kLogits = 0,  // Z = Xhat W^T (A: Xhat K-major, B: W K-major); epilogue: per-tile
+                //   max / sum of exp, target logit, bf16 exp(z - tile max) stored
+  kDxhat = 1,   // dXhat = G W (A: G K-major, B: W MN-major); epilogue: fp32 store
+  kDW = 2       // dW = G^T Xhat over the final module (A: G MN-major,
+                //   B: Xhat MN-major); epilogue: fp32 store
+};
+
+struct GemmArgs {
+  int32_t M;          // rows of the product
+  int32_t N;          // columns of the product
+  int32_t k_blocks;   // reduction length / kBK, rounded up
+  int32_t k_row0;     // first reduction row in A/B coordinates (kDW: first token of the module)
+  int32_t m_blocks;
+  int32_t n_blocks;
+  int32_t group_m;    // tile raster: group_m row blocks sweep all column blocks together
+  int32_t num_tiles;
+  // kLogits epilogue
+  const int32_t* targets;  // [M] token targets (flattened [K, N])
+  float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile
+  float* zy;               // [M]: logit of the target
+  int32_t V;
+  uint32_t* flags;         // device flag word
+};
+
+size_t gemm_smem_bytes();
+cudaError_t gemm_prepare(int device);  // sets the dynamic shared memory limit once per device
+cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
+                        const CUtensorMap& d, const GemmArgs& args, int grid,
+                        cudaStream_t stream);
+
+// ---- row kernels ---------------------------------------------------------------
+
+constexpr int kMaxModules = 16;
+
+struct RowArgs {
+  const uint16_t* hidden[kMaxModules];
+  uint16_t* dhidden[kMaxModules];
+  int64_t N;
+  int32_t K;
+  int32_t d;
+  int32_t V;
+  int32_t ldp;          // row stride (elements) of the exponential / gradient buffer
+  int32_t n_tiles_v;    // column tiles of the logits product
+  int32_t ignore_index;
+  float eps;
+  const uint16_t* gamma;
+  const int32_t* targets;
+  const uint8_t* mask;
+  float* r;             // [M]
+  uint16_t* xhat;       // [M, d]
+  float* lse;           // [M]
+  float* zy;            // [M]
+  float2* stats;        // [n_tiles_v, M]
+  double* part_sum;     // [K, part_blocks]
+  int32_t* part_cnt;    // [K, part_blocks]
+  int32_t part_blocks;
+  float* inv_nvalid;    // [K]
+  float* loss_tok;      // [K, N] or null
+  float* loss_mean;     // [K]
+  uint16_t* P;          // [M, ldp] bf16: exp(z - tile max), turned into G in place
+  float* dxhat;         // [M, d]
+  float* dgamma_part;   // [dg_chunks, d]
+  int32_t dg_chunks;
+  int32_t dg_rows;      // rows per dgamma chunk
+  float* dgamma;        // [d] or null
+  uint32_t* flags;
+};
+
+cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s);
+cudaError_t launch_lse(const RowArgs& a, cudaStream_t s);
+cudaError_t launch_grad(const RowArgs& a, cudaStream_t s);
+cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts);
+cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s);
+
+}  // namespace solo

@@ -1,0 +1,313 @@
+// Row-wise kernels of the readout path: the final RMSNorm and its backward,
+// the log-sum-exp combination of per-tile statistics with the token loss and
+// module means, the gradient of the logits, and the dgamma reduction.
+//
+// All reductions run in a fixed order (no floating-point atomics), so every
+// output is bitwise reproducible from run to run.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "../../include/solo_readout.h"
+
+namespace solo {
+namespace {
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&b);
+}
+
+__device__ __forceinline__ void unpack8(const uint4& x, float (&f)[8]) {
+  f[0] = bf16_lo(x.x); f[1] = bf16_hi(x.x);
+  f[2] = bf16_lo(x.y); f[3] = bf16_hi(x.y);
+  f[4] = bf16_lo(x.z); f[5] = bf16_hi(x.z);
+  f[6] = bf16_lo(x.w); f[7] = bf16_hi(x.w);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ bool token_kept(const RowArgs& a, int64_t row, int y) {
+  const bool in_range = y >= 0 && y < a.V;
+  return in_range && y != a.ignore_index && (a.mask == nullptr || a.mask[row] != 0);
+}
+
+// ---- final RMSNorm: r_i = (mean_j h_ij^2 + eps)^-1/2, xhat = bf16(gamma h r) ------
+
+__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (row >= M) return;
+  const int k = static_cast<int>(row / a.N);
+  const int64_t n = row - static_cast<int64_t>(k) * a.N;
+  const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
+  const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
+  const int nv = a.d / 8;
+  float ss = 0.f;
+  for (int v = lane; v < nv; v += 32) {
+    float f[8];
+    unpack8(__ldg(h + v), f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) ss = fmaf(f[j], f[j], ss);
+  }
+  ss = warp_sum(ss);
+  const float r = 1.0f / sqrtf(ss / static_cast<float>(a.d) + a.eps);
+  uint4* out = reinterpret_cast<uint4*>(a.xhat + row * a.d);
+  for (int v = lane; v < nv; v += 32) {
+    float f[8], gg[8];
+    unpack8(__ldg(h + v), f);
+    unpack8(__ldg(g + v), gg);
+    uint4 o;
+    // gamma * h is exact in fp32 (8 x 8 significant bits); one rounding for * r.
+    o.x = pack2(gg[0] * f[0] * r, gg[1] * f[1] * r);
+    o.y = pack2(gg[2] * f[2] * r, gg[3] * f[3] * r);
+    o.z = pack2(gg[4] * f[4] * r, gg[5] * f[5] * r);
+    o.w = pack2(gg[6] * f[6] * r, gg[7] * f[7] * r);
+    out[v] = o;
+  }
+  if (lane == 0) a.r[row] = r;
+}
+
+// ---- log-sum-exp over column tiles, token loss, per-block module sums ----------
+
+__global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
+  const int k = blockIdx.y;
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const int64_t n = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+  double lsum = 0.0;
+  int cnt = 0;
+  int bad = 0;
+  if (n < a.N) {
+    const int64_t row = static_cast<int64_t>(k) * a.N + n;
+    float mx = -INFINITY, s = 0.f;
+    for (int t = 0; t < a.n_tiles_v; ++t) {
+      const float2 st = a.stats[static_cast<int64_t>(t) * M + row];
+      if (st.x > mx) {
+        s = s * expf(mx - st.x) + st.y;
+        mx = st.x;
+      } else {
+        s += st.y * expf(st.x - mx);
+      }
+    }
+    const float l = mx + logf(s);
+    a.lse[row] = l;
+    const int y = a.targets[row];
+    bad = !(y >= 0 && y < a.V) && y != a.ignore_index;
+    const bool kept = token_kept(a, row, y);
+    const float loss = kept ? l - a.zy[row] : 0.f;
+    if (a.loss_tok) a.loss_tok[row] = loss;
+    lsum = loss;
+    cnt = kept ? 1 : 0;
+  }
+  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(a.flags, SOLO_FLAG_BAD_TARGET);
+  __shared__ double ssum[8];
+  __shared__ int scnt[8];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+    cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    ssum[threadIdx.x >> 5] = lsum;
+    scnt[threadIdx.x >> 5] = cnt;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    int c = 0;
+    for (int w = 0; w < 8; ++w) {
+      t += ssum[w];
+      c += scnt[w];
+    }
+    a.part_sum[static_cast<int64_t>(k) * a.part_blocks + blockIdx.x] = t;
+    a.part_cnt[static_cast<int64_t>(k) * a.part_blocks + blockIdx.x] = c;
+  }
+}
+
+__global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
+  const int k = blockIdx.x;
+  double t = 0.0;
+  long long c = 0;
+  for (int b = threadIdx.x; b < a.part_blocks; b += 256) {
+    t += a.part_sum[static_cast<int64_t>(k) * a.part_blocks + b];
+    c += a.part_cnt[static_cast<int64_t>(k) * a.part_blocks + b];
+  }
+  __shared__ double st[256];
+  __shared__ long long sc[256];
+  st[threadIdx.x] = t;
+  sc[threadIdx.x] = c;
+  __syncthreads();
+  for (int o = 128; o > 0; o >>= 1) {
+    if (threadIdx.x < o) {
+      st[threadIdx.x] += st[threadIdx.x + o];
+      sc[threadIdx.x] += sc[threadIdx.x + o];
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const long long nv = sc[0];
+    a.loss_mean[k] = nv > 0 ? static_cast<float>(st[0] / static_cast<double>(nv)) : 0.f;
+    a.inv_nvalid[k] = nv > 0 ? static_cast<float>(1.0 / static_cast<double>(nv)) : 0.f;
+  }
+}
+
+// ---- dL/dz in place: G = (softmax - onehot) / Nvalid --------------------------
+// The buffer holds p~ = bf16(exp(z - m_t)) for the column tile t of each
+// entry, so softmax = p~ * exp(m_t - lse).  The target entry is recomputed
+// from the fp32 target logit so that p_y - 1 keeps its relative precision.
+
+__global__ void __launch_bounds__(256) grad_kernel(const RowArgs a) {
+  extern __shared__ float ctile[];
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const int64_t row = blockIdx.x;
+  const int k = static_cast<int>(row / a.N);
+  const int y = a.targets[row];
+  uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
+  const int nvec = a.ldp / 8;
+  if (!token_kept(a, row, y)) {
+    for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  const float w = a.inv_nvalid[k];
+  const float l = a.lse[row];
+  for (int t = threadIdx.x; t < a.n_tiles_v; t += 256)
+    ctile[t] = expf(a.stats[static_cast<int64_t>(t) * M + row].x - l) * w;
+  const float gy = (expf(a.zy[row] - l) - 1.0f) * w;
+  __syncthreads();
+  for (int v = threadIdx.x; v < nvec; v += 256) {
+    const int v0 = v * 8;
+    if (v0 >= a.V) {
+      P[v] = make_uint4(0, 0, 0, 0);
+      continue;
+    }
+    const float c = ctile[v0 / kBN];
+    float f[8];
+    unpack8(P[v], f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      f[j] *= c;
+      if (v0 + j >= a.V) f[j] = 0.f;
+      if (v0 + j == y) f[j] = gy;
+    }
+    P[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+  }
+}
+
+// ---- RMSNorm backward: dh = r gamma dxhat - (r^3/d) h sum_l gamma_l dxhat_l h_l --
+
+__global__ void __launch_bounds__(256) norm_bwd_kernel(const RowArgs a) {
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (row >= M) return;
+  const int k = static_cast<int>(row / a.N);
+  const int64_t n = row - static_cast<int64_t>(k) * a.N;
+  const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
+  const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
+  const float4* dx = reinterpret_cast<const float4*>(a.dxhat + row * a.d);
+  const int nv = a.d / 8;
+  float c = 0.f;
+  for (int v = lane; v < nv; v += 32) {
+    float f[8], gg[8];
+    unpack8(__ldg(h + v), f);
+    unpack8(__ldg(g + v), gg);
+    const float4 d0 = dx[2 * v], d1 = dx[2 * v + 1];
+    c = fmaf(gg[0] * d0.x, f[0], c); c = fmaf(gg[1] * d0.y, f[1], c);
+    c = fmaf(gg[2] * d0.z, f[2], c); c = fmaf(gg[3] * d0.w, f[3], c);
+    c = fmaf(gg[4] * d1.x, f[4], c); c = fmaf(gg[5] * d1.y, f[5], c);
+    c = fmaf(gg[6] * d1.z, f[6], c); c = fmaf(gg[7] * d1.w, f[7], c);
+  }
+  c = warp_sum(c);
+  const float r = a.r[row];
+  const float coef = r * r * r * c / static_cast<float>(a.d);
+  uint4* out = reinterpret_cast<uint4*>(a.dhidden[k] + n * a.d);
+  for (int v = lane; v < nv; v += 32) {
+    float f[8], gg[8];
+    unpack8(__ldg(h + v), f);
+    unpack8(__ldg(g + v), gg);
+    const float4 d0 = dx[2 * v], d1 = dx[2 * v + 1];
+    const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+    float o[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = fmaf(r * gg[j], dd[j], -coef * f[j]);
+    out[v] = make_uint4(pack2(o[0], o[1]), pack2(o[2], o[3]), pack2(o[4], o[5]), pack2(o[6], o[7]));
+  }
+}
+
+// ---- dgamma of the final module: sum_i dxhat_ij h_ij r_i, two fixed-order stages --
+
+__global__ void __launch_bounds__(256) dgamma_part_kernel(const RowArgs a) {
+  const int j = blockIdx.x * 256 + threadIdx.x;
+  const int chunk = blockIdx.y;
+  if (j >= a.d) return;
+  const int k = a.K - 1;
+  const int64_t n0 = static_cast<int64_t>(chunk) * a.dg_rows;
+  const int64_t n1 = min(a.N, n0 + a.dg_rows);
+  const uint16_t* h = a.hidden[k];
+  const int64_t row0 = static_cast<int64_t>(k) * a.N;
+  float acc = 0.f;
+  for (int64_t n = n0; n < n1; ++n) {
+    const float hv = __uint_as_float(static_cast<uint32_t>(h[n * a.d + j]) << 16);
+    acc = fmaf(a.dxhat[(row0 + n) * a.d + j] * a.r[row0 + n], hv, acc);
+  }
+  a.dgamma_part[static_cast<int64_t>(chunk) * a.d + j] = acc;
+}
+
+__global__ void __launch_bounds__(256) dgamma_reduce_kernel(const RowArgs a) {
+  const int j = blockIdx.x * 256 + threadIdx.x;
+  if (j >= a.d) return;
+  float acc = 0.f;
+  for (int c = 0; c < a.dg_chunks; ++c) acc += a.dgamma_part[static_cast<int64_t>(c) * a.d + j];
+  a.dgamma[j] = acc;
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  rmsnorm_fwd_kernel<<<static_cast<unsigned>((M + 7) / 8), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lse(const RowArgs& a, cudaStream_t s) {
+  lse_kernel<<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  module_mean_kernel<<<a.K, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const size_t smem = static_cast<size_t>(a.n_tiles_v) * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  grad_kernel<<<static_cast<unsigned>(M), 256, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts) {
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  norm_bwd_kernel<<<static_cast<unsigned>((M + 7) / 8), 256, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !want_dgamma_parts) return e;
+  dgamma_part_kernel<<<dim3((a.d + 255) / 256, a.dg_chunks), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s) {
+  dgamma_reduce_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace solo

@@ -1,0 +1,368 @@
+// Host side of the C ABI: argument checks, workspace layout, TMA tensor maps
+// and the launch sequence of one call.
+//
+// Launch sequence (all on the caller's stream, no host synchronisation):
+//   rmsnorm      r_i and xhat = bf16(gamma h r)                  [K*N, d]
+//   logits       tensor-core xhat W^T; per (row, 256-column tile) max and
+//                sum of exp, target logit, bf16 exp(z - tile max)  [K*N, V]
+//   lse          log-sum-exp per row, token loss, module means, 1/Nvalid
+//   grad         (softmax - onehot)/Nvalid in place, bf16        [K*N, V]
+//   dxhat        tensor-core G W, fp32                            [K*N, d]
+//   norm_bwd     dH through the RMSNorm Jacobian, dgamma partial sums
+//   dW           tensor-core G^T xhat over the final module       [V, d]
+//   dgamma       fixed-order sum of the partials                  [d]
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/solo_readout.h"
+#include "internal.h"
+
+namespace {
+
+using namespace solo;
+
+constexpr size_t kAlign = 1024;
+constexpr int kDgRows = 64;
+constexpr int kGroupM = 16;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Layout {
+  int64_t M = 0;
+  int ldp = 0;
+  int n_tiles_v = 0;
+  int part_blocks = 0;
+  int dg_chunks = 0;
+  size_t flags = 0, r = 0, lse = 0, zy = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
+  size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0, total = 0;
+};
+
+solo_status_t check_dims(const solo_dims_t* d) {
+  if (d == nullptr) return SOLO_ERR_INVALID_ARG;
+  if (d->K < 1 || d->K > SOLO_MAX_MODULES) return SOLO_ERR_INVALID_ARG;
+  if (d->N < 1 || d->d < 8 || d->V < 1) return SOLO_ERR_INVALID_ARG;
+  if (!(d->eps >= 0.0f) || !std::isfinite(d->eps)) return SOLO_ERR_INVALID_ARG;
+  if (d->d % 8 != 0) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  // row and column coordinates of the tensor-core operands are 32-bit
+  const int64_t M = static_cast<int64_t>(d->K) * d->N;
+  if (M > (int64_t{1} << 31) - 1 - kBM) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  if (d->V > (1 << 30) || d->d > (1 << 20)) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  return SOLO_OK;
+}
+
+Layout make_layout(const solo_dims_t& d) {
+  Layout L;
+  L.M = static_cast<int64_t>(d.K) * d.N;
+  L.ldp = static_cast<int>(align_up(d.V, 8));
+  L.n_tiles_v = (d.V + kBN - 1) / kBN;
+  L.part_blocks = static_cast<int>((d.N + 255) / 256);
+  L.dg_chunks = static_cast<int>((d.N + kDgRows - 1) / kDgRows);
+  const size_t M = static_cast<size_t>(L.M);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes, kAlign);
+    return at;
+  };
+  L.flags = take(256);
+  L.r = take(M * 4);
+  L.lse = take(M * 4);
+  L.zy = take(M * 4);
+  L.part_sum = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
+  L.part_cnt = take(static_cast<size_t>(d.K) * L.part_blocks * 4);
+  L.inv_nvalid = take(SOLO_MAX_MODULES * 4);
+  L.stats = take(static_cast<size_t>(L.n_tiles_v) * M * 8);
+  L.xhat = take(M * d.d * 2);
+  L.P = take(M * static_cast<size_t>(L.ldp) * 2);
+  L.dxhat = take(M * d.d * 4);
+  L.dgp = take(static_cast<size_t>(L.dg_chunks) * d.d * 4);
+  L.total = off;
+  return L;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ---- per-device setup ------------------------------------------------------------
+
+struct DeviceInfo {
+  bool ready = false;
+  bool sm103 = false;
+  int sms = 0;
+};
+
+std::mutex g_dev_mu;
+DeviceInfo g_dev[64];
+
+solo_status_t device_setup(int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SOLO_ERR_CUDA;
+  if (dev < 0 || dev >= 64) return SOLO_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  DeviceInfo& info = g_dev[dev];
+  if (!info.ready) {
+    int major = 0, minor = 0, sms_ = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms_, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return SOLO_ERR_CUDA;
+    info.sm103 = (major == 10 && minor == 3);
+    info.sms = sms_;
+    if (info.sm103 && gemm_prepare(dev) != cudaSuccess) return SOLO_ERR_CUDA;
+    info.ready = true;
+  }
+  if (!info.sm103) return SOLO_ERR_NOT_SM103;
+  *sms = info.sms;
+  return SOLO_OK;
+}
+
+// ---- TMA tensor maps ----------------------------------------------------------------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D row-major tensor [outer, inner] with a row pitch of row_bytes, loaded
+// or stored in boxes of [box_outer, box_inner] with 128-byte swizzle; reads
+// outside the tensor return zeros and writes outside it are dropped.
+bool make_map(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t inner,
+              uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, dt, 2, const_cast<void*>(ptr), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                  const solo_bf16_t* gamma, const solo_bf16_t* W, const int32_t* targets,
+                  const uint8_t* mask, float* loss_tok, float* loss_mean,
+                  solo_bf16_t* const* dhidden, float* dW, float* dgamma, void* workspace,
+                  size_t workspace_bytes, cudaStream_t stream, void* const* events,
+                  int32_t n_events) {
+  // -------- host-side checks: nothing is enqueued when one fails
+  solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  const solo_dims_t& D = *dims;
+  if (hidden == nullptr || dhidden == nullptr || gamma == nullptr || W == nullptr ||
+      targets == nullptr || loss_mean == nullptr || workspace == nullptr)
+    return SOLO_ERR_INVALID_ARG;
+  if (events != nullptr && n_events != SOLO_NUM_STAGES + 1) return SOLO_ERR_INVALID_ARG;
+  for (int k = 0; k < D.K; ++k) {
+    if (hidden[k] == nullptr || dhidden[k] == nullptr) return SOLO_ERR_INVALID_ARG;
+    if (!aligned16(hidden[k]) || !aligned16(dhidden[k])) return SOLO_ERR_MISALIGNED;
+  }
+  if (!aligned16(gamma) || !aligned16(W) || !aligned16(workspace) ||
+      (reinterpret_cast<uintptr_t>(targets) & 3u) || (dW && !aligned16(dW)) ||
+      (dgamma && (reinterpret_cast<uintptr_t>(dgamma) & 3u)) ||
+      (loss_tok && (reinterpret_cast<uintptr_t>(loss_tok) & 3u)) ||
+      (reinterpret_cast<uintptr_t>(loss_mean) & 3u))
+    return SOLO_ERR_MISALIGNED;
+  const Layout L = make_layout(D);
+  if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+
+  // -------- device
+  int sms = 0;
+  st = device_setup(&sms);
+  if (st != SOLO_OK) return st;
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  RowArgs ra;
+  std::memset(&ra, 0, sizeof(ra));
+  for (int k = 0; k < D.K; ++k) {
+    ra.hidden[k] = hidden[k];
+    ra.dhidden[k] = dhidden[k];
+  }
+  ra.N = D.N;
+  ra.K = D.K;
+  ra.d = D.d;
+  ra.V = D.V;
+  ra.ldp = L.ldp;
+  ra.n_tiles_v = L.n_tiles_v;
+  ra.ignore_index = D.ignore_index;
+  ra.eps = D.eps;
+  ra.gamma = gamma;
+  ra.targets = targets;
+  ra.mask = mask;
+  ra.r = reinterpret_cast<float*>(ws + L.r);
+  ra.xhat = reinterpret_cast<uint16_t*>(ws + L.xhat);
+  ra.lse = reinterpret_cast<float*>(ws + L.lse);
+  ra.zy = reinterpret_cast<float*>(ws + L.zy);
+  ra.stats = reinterpret_cast<float2*>(ws + L.stats);
+  ra.part_sum = reinterpret_cast<double*>(ws + L.part_sum);
+  ra.part_cnt = reinterpret_cast<int32_t*>(ws + L.part_cnt);
+  ra.part_blocks = L.part_blocks;
+  ra.inv_nvalid = reinterpret_cast<float*>(ws + L.inv_nvalid);
+  ra.loss_tok = loss_tok;
+  ra.loss_mean = loss_mean;
+  ra.P = reinterpret_cast<uint16_t*>(ws + L.P);
+  ra.dxhat = reinterpret_cast<float*>(ws + L.dxhat);
+  ra.dgamma_part = reinterpret_cast<float*>(ws + L.dgp);
+  ra.dg_chunks = L.dg_chunks;
+  ra.dg_rows = kDgRows;
+  ra.dgamma = dgamma;
+  ra.flags = reinterpret_cast<uint32_t*>(ws + L.flags);
+
+  const uint64_t M = static_cast<uint64_t>(L.M);
+  const uint64_t d = static_cast<uint64_t>(D.d);
+  const uint64_t V = static_cast<uint64_t>(D.V);
+  const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+  CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW;
+  bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, kBK, kBM) &&
+            make_map(&mW_k, BF, W, d, V, d * 2, kBK, kBN) &&
+            make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
+            make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, kBK, kBM) &&
+            make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK) &&
+            make_map(&mDX, F32, ra.dxhat, d, M, d * 4, 32, 32);
+  if (ok && dW) {
+    ok = make_map(&mG_mn, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBK) &&
+         make_map(&mX_mn, BF, ra.xhat, d, M, d * 2, 64, kBK) &&
+         make_map(&mDW, F32, dW, d, V, d * 4, 32, 32);
+  }
+  if (!ok) return SOLO_ERR_CUDA;
+
+  auto mark = [&](int stage) -> bool {
+    if (events == nullptr) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(events[stage]), stream) == cudaSuccess;
+  };
+  auto fail = [](cudaError_t e) { return e != cudaSuccess; };
+
+  if (fail(cudaMemsetAsync(ra.flags, 0, 256, stream))) return SOLO_ERR_CUDA;
+
+  if (!mark(SOLO_STAGE_RMSNORM) || fail(launch_rmsnorm_fwd(ra, stream))) return SOLO_ERR_CUDA;
+
+  GemmArgs g;
+  std::memset(&g, 0, sizeof(g));
+  g.M = static_cast<int32_t>(M);
+  g.N = D.V;
+  g.k_blocks = static_cast<int32_t>((d + kBK - 1) / kBK);
+  g.k_row0 = 0;
+  g.m_blocks = static_cast<int32_t>((M + kBM - 1) / kBM);
+  g.n_blocks = L.n_tiles_v;
+  g.group_m = kGroupM;
+  g.num_tiles = g.m_blocks * g.n_blocks;
+  g.targets = targets;
+  g.stats = ra.stats;
+  g.zy = ra.zy;
+  g.V = D.V;
+  g.flags = ra.flags;
+  if (!mark(SOLO_STAGE_LOGITS) ||
+      fail(launch_gemm(kLogits, mX_k, mW_k, mP_st, g, std::min(g.num_tiles, sms), stream)))
+    return SOLO_ERR_CUDA;
+
+  if (!mark(SOLO_STAGE_LSE) || fail(launch_lse(ra, stream))) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_STAGE_GRAD) || fail(launch_grad(ra, stream))) return SOLO_ERR_CUDA;
+
+  GemmArgs gx = g;
+  gx.N = D.d;
+  gx.k_blocks = (D.V + kBK - 1) / kBK;
+  gx.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
+  gx.num_tiles = gx.m_blocks * gx.n_blocks;
+  if (!mark(SOLO_STAGE_DXHAT) ||
+      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, gx, std::min(gx.num_tiles, sms), stream)))
+    return SOLO_ERR_CUDA;
+
+  if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_norm_bwd(ra, stream, dgamma != nullptr)))
+    return SOLO_ERR_CUDA;
+
+  if (!mark(SOLO_STAGE_DW)) return SOLO_ERR_CUDA;
+  if (dW) {
+    GemmArgs gw = g;
+    gw.M = D.V;
+    gw.N = D.d;
+    gw.k_blocks = static_cast<int32_t>((D.N + kBK - 1) / kBK);
+    gw.k_row0 = static_cast<int32_t>(static_cast<int64_t>(D.K - 1) * D.N);
+    gw.m_blocks = (D.V + kBM - 1) / kBM;
+    gw.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
+    gw.num_tiles = gw.m_blocks * gw.n_blocks;
+    if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, gw, std::min(gw.num_tiles, sms), stream)))
+      return SOLO_ERR_CUDA;
+  }
+  if (!mark(SOLO_STAGE_DGAMMA)) return SOLO_ERR_CUDA;
+  if (dgamma && fail(launch_dgamma_reduce(ra, stream))) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_NUM_STAGES)) return SOLO_ERR_CUDA;
+  return SOLO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes) {
+  if (bytes == nullptr) return SOLO_ERR_INVALID_ARG;
+  const solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  *bytes = make_layout(*dims).total;
+  return SOLO_OK;
+}
+
+solo_status_t solo_readout_fwd_bwd(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                                   const solo_bf16_t* gamma, const solo_bf16_t* W,
+                                   const int32_t* targets, const uint8_t* mask, float* loss_tok,
+                                   float* loss_mean, solo_bf16_t* const* dhidden, float* dW,
+                                   float* dgamma, void* workspace, size_t workspace_bytes,
+                                   solo_stream_t stream) {
+  return run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
+             workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), nullptr, 0);
+}
+
+solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
+                                          const solo_bf16_t* const* hidden,
+                                          const solo_bf16_t* gamma, const solo_bf16_t* W,
+                                          const int32_t* targets, const uint8_t* mask,
+                                          float* loss_tok, float* loss_mean,
+                                          solo_bf16_t* const* dhidden, float* dW, float* dgamma,
+                                          void* workspace, size_t workspace_bytes,
+                                          solo_stream_t stream, void* const* events,
+                                          int32_t n_events) {
+  if (events == nullptr) return SOLO_ERR_INVALID_ARG;
+  return run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
+             workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), events,
+             n_events);
+}
+
+solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream,
+                                     uint32_t* flags) {
+  if (workspace == nullptr || flags == nullptr) return SOLO_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t v = 0;
+  if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return SOLO_ERR_CUDA;
+  *flags = v;
+  return SOLO_OK;
+}
+
+const char* solo_readout_strerror(solo_status_t status) {
+  switch (status) {
+    case SOLO_OK: return "success";
+    case SOLO_ERR_INVALID_ARG: return "invalid argument (NULL pointer or dims out of range)";
+    case SOLO_ERR_UNSUPPORTED_SHAPE: return "unsupported shape (d must be a multiple of 8)";
+    case SOLO_ERR_WORKSPACE_TOO_SMALL: return "workspace smaller than solo_readout_workspace_bytes";
+    case SOLO_ERR_CUDA: return "a CUDA runtime call failed";
+    case SOLO_ERR_NOT_SM103: return "current device is not compute capability 10.3 (sm_103a)";
+    case SOLO_ERR_MISALIGNED: return "a tensor pointer is not suitably aligned (16 bytes)";
+    default: return "unknown status";
+  }
+}
+
+int32_t solo_readout_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,198 @@
+"""Thin ctypes binding of libsolo_readout (argument marshalling only).
+
+Function names match the C ABI in ``include/solo_readout.h``.  Tensors are
+PyTorch tensors used for device memory and streams: their data pointers and
+the current CUDA stream are handed to the library; every step of the
+computation runs in the library's kernels.  There is no fallback: when the
+library is missing or the device is not sm_103a the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Sequence
+
+from . import build as _build
+
+SOLO_OK = 0
+SOLO_ERR_INVALID_ARG = -1
+SOLO_ERR_UNSUPPORTED_SHAPE = -2
+SOLO_ERR_WORKSPACE_TOO_SMALL = -3
+SOLO_ERR_CUDA = -4
+SOLO_ERR_NOT_SM103 = -5
+SOLO_ERR_MISALIGNED = -6
+
+SOLO_FLAG_BAD_TARGET = 1
+SOLO_FLAG_TIMEOUT = 2
+
+SOLO_NUM_STAGES = 8
+STAGE_NAMES = ["rmsnorm", "logits", "lse", "grad", "dxhat", "norm_bwd", "dW", "dgamma"]
+
+
+class solo_dims_t(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("N", ctypes.c_int64), ("d", ctypes.c_int32),
+                ("V", ctypes.c_int32), ("eps", ctypes.c_float),
+                ("ignore_index", ctypes.c_int32)]
+
+
+class SoloError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {strerror(status)} (status {status})")
+        self.status = status
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Loads the in-tree library (raises when it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or library_path()
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with "
+                          "`python -m paper_2609_35440_gb300.build` (needs nvcc)")
+    lib = ctypes.CDLL(path)
+    vp, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    dims_p = ctypes.POINTER(solo_dims_t)
+    lib.solo_readout_workspace_bytes.argtypes = [dims_p, ctypes.POINTER(sz)]
+    lib.solo_readout_workspace_bytes.restype = i32
+    common = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp, vp, vp, ctypes.POINTER(vp), vp, vp,
+              vp, sz, vp]
+    lib.solo_readout_fwd_bwd.argtypes = common
+    lib.solo_readout_fwd_bwd.restype = i32
+    lib.solo_readout_fwd_bwd_events.argtypes = common + [ctypes.POINTER(vp), i32]
+    lib.solo_readout_fwd_bwd_events.restype = i32
+    lib.solo_readout_get_flags.argtypes = [vp, vp, ctypes.POINTER(ctypes.c_uint32)]
+    lib.solo_readout_get_flags.restype = i32
+    lib.solo_readout_strerror.argtypes = [i32]
+    lib.solo_readout_strerror.restype = ctypes.c_char_p
+    lib.solo_readout_version.argtypes = []
+    lib.solo_readout_version.restype = i32
+    _lib = lib
+    return lib
+
+
+def strerror(status: int) -> str:
+    return load().solo_readout_strerror(int(status)).decode()
+
+
+def make_dims(K: int, N: int, d: int, V: int, eps: float = 1e-6,
+              ignore_index: int = -100) -> solo_dims_t:
+    return solo_dims_t(K, N, d, V, eps, ignore_index)
+
+
+def solo_readout_workspace_bytes(dims: solo_dims_t) -> int:
+    out = ctypes.c_size_t(0)
+    st = load().solo_readout_workspace_bytes(ctypes.byref(dims), ctypes.byref(out))
+    if st != SOLO_OK:
+        raise SoloError(st, "solo_readout_workspace_bytes")
+    return out.value
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    return t.data_ptr() if hasattr(t, "data_ptr") else int(t)
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _call(fn, dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
+          workspace, workspace_bytes, stream, extra=()):
+    K = dims.K
+    if len(hidden) != K or len(dhidden) != K:
+        raise ValueError("hidden and dhidden need K entries")
+    harr = (ctypes.c_void_p * K)(*[_ptr(h) for h in hidden])
+    darr = (ctypes.c_void_p * K)(*[_ptr(h) for h in dhidden])
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    st = fn(ctypes.byref(dims), harr, _ptr(gamma), _ptr(W), _ptr(targets), _ptr(mask),
+            _ptr(loss_tok), _ptr(loss_mean), darr, _ptr(dW), _ptr(dgamma), _ptr(workspace),
+            int(workspace_bytes), _stream_handle(stream), *extra)
+    return st
+
+
+def solo_readout_fwd_bwd(dims: solo_dims_t, hidden: Sequence, gamma, W, targets, mask,
+                         loss_tok, loss_mean, dhidden: Sequence, dW, dgamma, workspace,
+                         workspace_bytes: int | None = None, stream=None,
+                         check: bool = True) -> int:
+    """Enqueues one forward + backward; returns the status (raises on error when check)."""
+    st = _call(load().solo_readout_fwd_bwd, dims, hidden, gamma, W, targets, mask, loss_tok,
+               loss_mean, dhidden, dW, dgamma, workspace, workspace_bytes, stream)
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd")
+    return st
+
+
+def solo_readout_fwd_bwd_events(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean,
+                                dhidden, dW, dgamma, workspace, events,
+                                workspace_bytes: int | None = None, stream=None,
+                                check: bool = True) -> int:
+    """As solo_readout_fwd_bwd, recording ``events`` (SOLO_NUM_STAGES + 1 torch.cuda.Event
+    with timing enabled) around the stages."""
+    handles = []
+    for e in events:
+        h = e.cuda_event if hasattr(e, "cuda_event") else int(e)
+        handles.append(h)
+    arr = (ctypes.c_void_p * len(handles))(*handles)
+    st = _call(load().solo_readout_fwd_bwd_events, dims, hidden, gamma, W, targets, mask,
+               loss_tok, loss_mean, dhidden, dW, dgamma, workspace, workspace_bytes, stream,
+               extra=(arr, len(handles)))
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd_events")
+    return st
+
+
+def solo_readout_get_flags(workspace, stream=None) -> int:
+    out = ctypes.c_uint32(0)
+    st = load().solo_readout_get_flags(_ptr(workspace), _stream_handle(stream), ctypes.byref(out))
+    if st != SOLO_OK:
+        raise SoloError(st, "solo_readout_get_flags")
+    return out.value
+
+
+def solo_readout_version() -> int:
+    return load().solo_readout_version()
+
+
+class Readout:
+    """Owns the output and workspace tensors for one problem size (torch, one device)."""
+
+    def __init__(self, K: int, N: int, d: int, V: int, eps: float = 1e-6,
+                 ignore_index: int = -100, want_loss_tok: bool = True, want_dW: bool = True,
+                 want_dgamma: bool = True, device=None):
+        import torch
+        self.dims = make_dims(K, N, d, V, eps, ignore_index)
+        dev = torch.device("cuda" if device is None else device)
+        nbytes = solo_readout_workspace_bytes(self.dims)
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.loss_tok = torch.empty(K, N, dtype=torch.float32, device=dev) if want_loss_tok else None
+        self.loss_mean = torch.empty(K, dtype=torch.float32, device=dev)
+        self.dhidden = [torch.empty(N, d, dtype=torch.bfloat16, device=dev) for _ in range(K)]
+        self.dW = torch.empty(V, d, dtype=torch.float32, device=dev) if want_dW else None
+        self.dgamma = torch.empty(d, dtype=torch.float32, device=dev) if want_dgamma else None
+
+    def __call__(self, hidden, gamma, W, targets, mask=None, stream=None, events=None):
+        if events is None:
+            solo_readout_fwd_bwd(self.dims, hidden, gamma, W, targets, mask, self.loss_tok,
+                                 self.loss_mean, self.dhidden, self.dW, self.dgamma,
+                                 self.workspace, stream=stream)
+        else:
+            solo_readout_fwd_bwd_events(self.dims, hidden, gamma, W, targets, mask,
+                                        self.loss_tok, self.loss_mean, self.dhidden, self.dW,
+                                        self.dgamma, self.workspace, events, stream=stream)
+        return self
+
+    def flags(self, stream=None) -> int:
+        return solo_readout_get_flags(self.workspace, stream)

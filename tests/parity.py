@@ -1,0 +1,119 @@
+"""Helpers of the GPU parity tests: upload seeded inputs, run the library,
+run the oracle on the same bytes and compare with the stated tolerances.
+
+Tolerances (per the headline specification of this path):
+  per-token loss   abs err <= 2e-3
+  module mean loss rel err <= 1e-4
+  dH, dW, dgamma   max_abs(gpu - oracle) / max_abs(oracle) <= 2e-2, and
+                   cosine similarity >= 0.9999
+The oracle runs in "contract" mode: xhat is rounded to bf16 exactly where
+the GPU rounds it; everything after is fp64.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle.solo_oracle as orc
+from paper_2609_35440_gb300 import synth
+
+LOSS_TOK_ABS = 2e-3
+LOSS_MEAN_REL = 1e-4
+GRAD_REL = 2e-2
+GRAD_COS = 0.9999
+
+
+def to_device_bf16(bits: np.ndarray, device="cuda"):
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16))
+    return t.to(device).view(torch.bfloat16)
+
+
+def bf16_tensor_to_f64(t) -> np.ndarray:
+    import torch
+    return orc.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16))
+
+
+def run_gpu(wl, inp: synth.Inputs, mask: np.ndarray | None = None, want_dW=True,
+            want_dgamma=True, want_loss_tok=True, targets: np.ndarray | None = None):
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    dev = torch.device("cuda")
+    hidden = [to_device_bf16(inp.hidden[k]) for k in range(wl.K)]
+    gamma = to_device_bf16(inp.gamma)
+    W = to_device_bf16(inp.W)
+    tg = inp.targets if targets is None else targets
+    tgt = torch.from_numpy(np.ascontiguousarray(tg, dtype=np.int32)).to(dev)
+    mk = None if mask is None else torch.from_numpy(np.ascontiguousarray(mask, np.uint8)).to(dev)
+    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index,
+                    want_loss_tok=want_loss_tok, want_dW=want_dW, want_dgamma=want_dgamma)
+    ro(hidden, gamma, W, tgt, mk)
+    flags = ro.flags()
+    torch.cuda.synchronize()
+    out = dict(loss_mean=ro.loss_mean.double().cpu().numpy(), flags=flags,
+               dhidden=[bf16_tensor_to_f64(x) for x in ro.dhidden])
+    if want_loss_tok:
+        out["loss_tok"] = ro.loss_tok.double().cpu().numpy()
+    if want_dW:
+        out["dW"] = ro.dW.double().cpu().numpy()
+    if want_dgamma:
+        out["dgamma"] = ro.dgamma.double().cpu().numpy()
+    out["_ro"] = ro
+    return out
+
+
+def oracle_full(wl, inp: synth.Inputs, mask=None, targets=None):
+    dec = orc.bf16_bits_to_f64
+    hidden = [dec(inp.hidden[k]) for k in range(wl.K)]
+    tg = inp.targets if targets is None else targets
+    return orc.solo_readout_fwd_bwd(hidden, dec(inp.gamma), dec(inp.W), tg.astype(np.int64),
+                                    mask, eps=wl.eps, ignore_index=wl.ignore_index,
+                                    contract=True)
+
+
+def max_rel(a, ref) -> float:
+    a, ref = np.asarray(a, np.float64), np.asarray(ref, np.float64)
+    den = np.max(np.abs(ref)) if ref.size else 0.0
+    num = np.max(np.abs(a - ref)) if ref.size else 0.0
+    if den == 0.0:
+        return float(num)
+    return float(num / den)
+
+
+def cosine(a, ref) -> float:
+    a, ref = np.ravel(np.asarray(a, np.float64)), np.ravel(np.asarray(ref, np.float64))
+    na, nr = np.linalg.norm(a), np.linalg.norm(ref)
+    if na == 0.0 and nr == 0.0:
+        return 1.0
+    return float(np.dot(a, ref) / (na * nr))
+
+
+def check_grad(name, a, ref, report):
+    mr, cs = max_rel(a, ref), cosine(a, ref)
+    report[name] = (mr, cs)
+    zero_ref = not np.any(ref)
+    if zero_ref:
+        assert np.max(np.abs(a)) <= 1e-6, (name, "reference is zero", np.max(np.abs(a)))
+        return
+    assert mr <= GRAD_REL, (name, "max rel err", mr)
+    assert cs >= GRAD_COS, (name, "cosine", cs)
+
+
+def compare_full(wl, gpu, ref, check_dW=True, check_dgamma=True):
+    """Element-by-element comparison of every output; returns the error report."""
+    rep = {}
+    lt_err = float(np.max(np.abs(gpu["loss_tok"] - ref["loss_tok"])))
+    rep["loss_tok_abs"] = lt_err
+    assert lt_err <= LOSS_TOK_ABS, ("loss_tok", lt_err)
+    for k in range(wl.K):
+        want = ref["loss_mean"][k]
+        got = gpu["loss_mean"][k]
+        if want == 0.0:
+            assert got == 0.0, ("loss_mean", k, got)
+        else:
+            assert abs(got - want) / abs(want) <= LOSS_MEAN_REL, ("loss_mean", k, got, want)
+        check_grad(f"dH[{k}]", gpu["dhidden"][k], ref["dhidden"][k], rep)
+    if check_dW:
+        check_grad("dW", gpu["dW"], ref["dW"], rep)
+    if check_dgamma:
+        check_grad("dgamma", gpu["dgamma"], ref["dgamma"], rep)
+    return rep

@@ -1,0 +1,127 @@
+"""The C ABI on a machine without a GPU: the library loads, exports every
+entry point the header declares, and rejects bad arguments on the host
+before any CUDA call is made."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "solo_readout.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(solo_readout_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for n in ("solo_readout_workspace_bytes", "solo_readout_fwd_bwd",
+              "solo_readout_fwd_bwd_events", "solo_readout_get_flags",
+              "solo_readout_strerror", "solo_readout_version"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(built_library):
+    lib = ctypes.CDLL(built_library)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+@pytest.fixture(scope="module")
+def sr(built_library):
+    from paper_2609_35440_gb300 import solo_readout
+    solo_readout.load(built_library)
+    return solo_readout
+
+
+def test_strerror_and_version(sr):
+    assert sr.strerror(0) == "success"
+    for code in range(-6, 0):
+        assert sr.strerror(code) and sr.strerror(code) != "unknown status"
+    assert sr.strerror(-99) == "unknown status"
+    assert sr.solo_readout_version() >= 100
+
+
+def test_workspace_query(sr):
+    dims = sr.make_dims(4, 8192, 2048, 32000)
+    b = sr.solo_readout_workspace_bytes(dims)
+    M = 4 * 8192
+    # xhat (bf16) + exponentials/gradient (bf16) + dxhat (fp32) dominate
+    assert b >= M * 2048 * 2 + M * 32000 * 2 + M * 2048 * 4
+    assert b < 1.05 * (M * 2048 * 2 + M * 32000 * 2 + M * 2048 * 4) + 64 * 2 ** 20
+    small = sr.solo_readout_workspace_bytes(sr.make_dims(1, 1, 8, 1))
+    assert 0 < small < 2 ** 20
+
+
+@pytest.mark.parametrize("K,N,d,V,want", [
+    (0, 16, 64, 100, -1), (17, 16, 64, 100, -1), (2, 0, 64, 100, -1), (2, 16, 0, 100, -1),
+    (2, 16, 64, 0, -1), (2, 16, 60, 100, -2), (2, 16, 4, 100, -1),
+])
+def test_workspace_query_rejects_bad_dims(sr, K, N, d, V, want):
+    out = ctypes.c_size_t(0)
+    st = sr.load().solo_readout_workspace_bytes(ctypes.byref(sr.make_dims(K, N, d, V)),
+                                                ctypes.byref(out))
+    assert st == want
+
+
+def _args(sr, K=2, N=16, d=64, V=100, **over):
+    fake = 1 << 20            # 16-byte aligned fake device addresses: never dereferenced
+    a = dict(dims=sr.make_dims(K, N, d, V), hidden=[fake] * K, gamma=fake, W=fake,
+             targets=fake, mask=None, loss_tok=None, loss_mean=fake, dhidden=[fake] * K,
+             dW=None, dgamma=None, workspace=fake, workspace_bytes=1 << 40, stream=0)
+    a.update(over)
+    return a
+
+
+@pytest.mark.parametrize("over,want", [
+    (dict(gamma=None), -1), (dict(W=None), -1), (dict(targets=None), -1),
+    (dict(loss_mean=None), -1), (dict(workspace=None), -1),
+    (dict(hidden=[1 << 20, None]), -1), (dict(dhidden=[None, 1 << 20]), -1),
+    (dict(W=(1 << 20) + 8), -6), (dict(hidden=[(1 << 20) + 2, 1 << 20]), -6),
+    (dict(workspace=(1 << 20) + 4), -6), (dict(dW=(1 << 20) + 8), -6),
+    (dict(workspace_bytes=1024), -3),
+])
+def test_fwd_bwd_rejects_bad_arguments_before_launch(sr, over, want):
+    a = _args(sr, **over)
+    st = sr.solo_readout_fwd_bwd(a["dims"], a["hidden"], a["gamma"], a["W"], a["targets"],
+                                 a["mask"], a["loss_tok"], a["loss_mean"], a["dhidden"],
+                                 a["dW"], a["dgamma"], a["workspace"],
+                                 workspace_bytes=a["workspace_bytes"], stream=a["stream"],
+                                 check=False)
+    assert st == want
+
+
+def test_fwd_bwd_rejects_bad_dims(sr):
+    for dims, want in [(sr.make_dims(0, 16, 64, 100), -1), (sr.make_dims(2, 16, 12, 100), -2),
+                       (sr.make_dims(2, 16, 64, 100, eps=-1.0), -1),
+                       (sr.make_dims(2, 16, 64, 100, eps=float("nan")), -1)]:
+        a = _args(sr, dims=dims)
+        st = sr.solo_readout_fwd_bwd(dims, a["hidden"][:dims.K] or [1 << 20],
+                                     a["gamma"], a["W"], a["targets"], None, None,
+                                     a["loss_mean"], a["dhidden"][:dims.K] or [1 << 20], None,
+                                     None, a["workspace"], workspace_bytes=1 << 40, stream=0,
+                                     check=False) if dims.K > 0 else \
+            sr.load().solo_readout_fwd_bwd(ctypes.byref(dims), None, None, None, None, None,
+                                           None, None, None, None, None, None, 0, None)
+        assert st == want
+
+
+def test_events_variant_needs_all_events(sr):
+    a = _args(sr)
+    arr = (ctypes.c_void_p * 3)(1, 2, 3)
+    st = sr._call(sr.load().solo_readout_fwd_bwd_events, a["dims"], a["hidden"], a["gamma"],
+                  a["W"], a["targets"], None, None, a["loss_mean"], a["dhidden"], None, None,
+                  a["workspace"], a["workspace_bytes"], 0, extra=(arr, 3))
+    assert st == -1
+
+
+def test_binding_has_no_fallback(tmp_path, monkeypatch):
+    """A missing library raises instead of silently computing elsewhere."""
+    from paper_2609_35440_gb300 import solo_readout
+    monkeypatch.setattr(solo_readout, "_lib", None)
+    with pytest.raises(ImportError):
+        solo_readout.load(str(tmp_path / "missing.so"))

@@ -1,0 +1,124 @@
+"""GPU parity against the fp64 oracle, element by element, on sizes the
+oracle finishes in seconds: the smallest workload, ragged shapes that leave
+partial tiles in every dimension, masks, bad targets, optional outputs and
+run-to-run determinism.  All calls go through the C ABI."""
+import numpy as np
+import pytest
+
+from paper_2609_35440_gb300 import synth, workloads
+from paper_2609_35440_gb300.workloads import Workload
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda(built_library):
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_35440_gb300 import solo_readout
+    solo_readout.load(built_library)
+
+
+def _case(wl, mask=None, targets=None, **kw):
+    inp = synth.generate(wl)
+    gpu = parity.run_gpu(wl, inp, mask=mask, targets=targets, **kw)
+    ref = parity.oracle_full(wl, inp, mask=mask, targets=targets)
+    return inp, gpu, ref
+
+
+def test_smallest_workload_full_parity():
+    wl = workloads.SMOKE
+    _, gpu, ref = _case(wl)
+    rep = parity.compare_full(wl, gpu, ref)
+    assert gpu["flags"] == 0
+    print("report", rep)
+
+
+RAGGED = [
+    Workload("ragged_k3_n200_d72_v1001", K=3, N=200, d=72, V=1001, seed=31, mask_frac=0.1,
+             row_scale=True),
+    Workload("ragged_k2_n130_d264_v517", K=2, N=130, d=264, V=517, seed=32, heavy_frac=0.02),
+    Workload("k1_n64_d128_v300", K=1, N=64, d=128, V=300, seed=33),
+    Workload("k4_n33_d136_v4100_zipf", K=4, N=33, d=136, V=4100, seed=34, targets="zipf",
+             mask_frac=0.2),
+    Workload("k2_n1_d8_v16", K=2, N=1, d=8, V=16, seed=35),
+    Workload("k2_n300_d512_v2500_heavy", K=2, N=300, d=512, V=2500, seed=36, heavy_frac=0.01,
+             row_scale=True, mask_frac=0.05),
+]
+
+
+@pytest.mark.parametrize("wl", RAGGED, ids=lambda w: w.name)
+def test_ragged_shapes(wl):
+    _, gpu, ref = _case(wl)
+    parity.compare_full(wl, gpu, ref)
+
+
+def test_mask_array_and_bad_targets():
+    wl = Workload("masked_k2_n160_d128_v700", K=2, N=160, d=128, V=700, seed=41)
+    inp = synth.generate(wl)
+    mask = synth.random_mask(7, wl.K, wl.N, 0.25)
+    tg = inp.targets.copy()
+    tg[0, 3] = wl.V           # out of range: masked and flagged
+    tg[1, 9] = -7             # negative, not ignore_index: masked and flagged
+    tg[1, 10] = wl.ignore_index
+    gpu = parity.run_gpu(wl, inp, mask=mask, targets=tg)
+    ref = parity.oracle_full(wl, inp, mask=mask, targets=tg)
+    assert ref["bad_target"]
+    assert gpu["flags"] & 1
+    parity.compare_full(wl, gpu, ref)
+    for k, n in ((0, 3), (1, 9), (1, 10)):
+        assert gpu["loss_tok"][k, n] == 0.0
+        assert not np.any(gpu["dhidden"][k][n])
+    for k in range(wl.K):
+        dead = mask[k] == 0
+        assert np.all(gpu["loss_tok"][k][dead] == 0.0)
+        assert not np.any(gpu["dhidden"][k][dead])
+
+
+def test_module_without_kept_tokens():
+    wl = Workload("allmasked_k2_n100_d64_v300", K=2, N=100, d=64, V=300, seed=42)
+    inp = synth.generate(wl)
+    tg = inp.targets.copy()
+    tg[1, :] = wl.ignore_index       # final module: nothing kept
+    gpu = parity.run_gpu(wl, inp, targets=tg)
+    ref = parity.oracle_full(wl, inp, targets=tg)
+    assert gpu["loss_mean"][1] == 0.0 and gpu["flags"] == 0
+    assert not np.any(gpu["dhidden"][1]) and not np.any(gpu["dW"]) and not np.any(gpu["dgamma"])
+    parity.compare_full(wl, gpu, ref)
+
+
+def test_optional_outputs_and_determinism():
+    wl = Workload("k3_n96_d192_v900", K=3, N=96, d=192, V=900, seed=43, mask_frac=0.1)
+    inp = synth.generate(wl)
+    a = parity.run_gpu(wl, inp)
+    b = parity.run_gpu(wl, inp)
+    for key in ("loss_tok", "loss_mean", "dW", "dgamma"):
+        assert np.array_equal(a[key], b[key]), key
+    for k in range(wl.K):
+        assert np.array_equal(a["dhidden"][k], b["dhidden"][k])
+    c = parity.run_gpu(wl, inp, want_dW=False, want_dgamma=False, want_loss_tok=False)
+    assert np.array_equal(a["loss_mean"], c["loss_mean"])
+    for k in range(wl.K):
+        assert np.array_equal(a["dhidden"][k], c["dhidden"][k])
+
+
+def test_workspace_reuse_across_shapes():
+    """A workspace sized for a larger problem serves a smaller one; stale contents do not leak."""
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    big = Workload("k2_n256_d256_v2048", K=2, N=256, d=256, V=2048, seed=44)
+    small = Workload("k2_n100_d128_v1000", K=2, N=100, d=128, V=1000, seed=45, mask_frac=0.1)
+    ws = torch.zeros(sr.solo_readout_workspace_bytes(sr.make_dims(big.K, big.N, big.d, big.V)),
+                     dtype=torch.uint8, device="cuda")
+    for wl in (big, small, big):
+        inp = synth.generate(wl)
+        gpu = parity.run_gpu(wl, inp)
+        ro = gpu["_ro"]
+        ro.workspace = ws
+        hid = [parity.to_device_bf16(inp.hidden[k]) for k in range(wl.K)]
+        ro(hid, parity.to_device_bf16(inp.gamma), parity.to_device_bf16(inp.W),
+           torch.from_numpy(inp.targets).cuda())
+        torch.cuda.synchronize()
+        assert torch.equal(ro.loss_mean.cpu(), torch.from_numpy(gpu["loss_mean"]).float())
