@@ -1,0 +1,424 @@
+"""Throughput of the SOLO shared-readout local loss (forward + backward) on GB300.
+
+One step = one call of solo_readout_fwd_bwd over all K modules: final
+RMSNorm, logits through the shared readout, softmax cross-entropy, dH for
+every module, dW and dgamma for the final module.  The default workload is
+the headline one: K=4 modules of N=8192 tokens, d=2048, V=32000.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints ONE JSON line (rank 0).  Under torchrun each rank runs an independent
+replica of the workload on its own GPU (the path has no exchange step), and
+the value is the tokens of all ranks over the slowest rank's time.
+
+Timing: inputs are resident in HBM; hidden states and W (265 MB) exceed the
+129 MB L2 and every step writes its 2.1 GB logit-gradient buffer, so no step
+finds its inputs in L2.  CUDA events on the launching stream, W >= 3 warm-up
+steps, a barrier and a device synchronize on both sides of the timed region.
+``e2e`` repeats the measurement through the same C ABI call with the step's
+inputs copied from pinned host memory and the losses read back, inside the
+timed region.  ``cpu_baseline`` times the fp64 oracle on a bounded sample
+of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_35440_gb300 import costmodel, synth, workloads  # noqa: E402
+
+METRIC = "local-readout CE fwd+bwd tokens/s at d=2048,V=32000; % of bf16 tensor peak"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNEL_SOURCES = ["paper_2609_35440_gb300/csrc/gemm_tc.cu", "paper_2609_35440_gb300/csrc/ptx.cuh",
+                  "paper_2609_35440_gb300/csrc/internal.h"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "logits_gemm_traffic.txt")
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default=workloads.HEADLINE.name,
+                   help="a workload name, or k<K>_n<N>_d<d>_v<V> for a custom uniform one")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    return p.parse_args()
+
+
+def workload_from_name(name: str) -> workloads.Workload:
+    if name in workloads.BY_NAME:
+        return workloads.BY_NAME[name]
+    import re
+    m = re.fullmatch(r"k(\d+)_n(\d+)_d(\d+)_v(\d+)", name)
+    if not m:
+        raise SystemExit(f"unknown workload {name}")
+    K, N, d, V = map(int, m.groups())
+    return workloads.Workload(name, K=K, N=N, d=d, V=V, seed=7)
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return FALLBACK_PEAKS, "fallback"
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(wl):
+    """Bytes per launch of the logits GEMM from the committed ncu capture, if the
+    kernel source is unchanged since; scaled by the tiles of this workload."""
+    try:
+        kv = {}
+        with open(TRAFFIC_FILE) as f:
+            for ln in f:
+                if "=" in ln and not ln.startswith("#"):
+                    k, v = ln.split("=", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("kernel_sha") != kernel_hash():
+            return None
+        per_unit = float(kv["dram_bytes_per_token_per_vocab_tile"])
+        return per_unit * wl.M * ((wl.V + 255) // 256) * (wl.d / float(kv["d"]))
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------- CPU legs
+
+def oracle_sample(wl, rows: int, inp_rows=None):
+    """One bounded oracle pass: the first `rows` tokens of every module, forward and
+    dH, plus dW/dgamma contributions of the final module's sampled rows."""
+    import oracle.solo_oracle as orc
+    if inp_rows is None:
+        inp_rows = prepare_oracle_sample(wl, rows)
+    hidden, gamma, W, targets = inp_rows
+    for k in range(wl.K):
+        y = targets[k].astype(np.int64)
+        kept, _ = orc.kept_tokens(y, None, wl.V, wl.ignore_index)
+        res = orc.module_rows(hidden[k], gamma, W, y, kept, max(int(kept.sum()), 1),
+                              float(np.float32(wl.eps)), True)
+        if k == wl.K - 1:
+            orc.readout_grads(res["g"], res["xhat"], res["dxhat"], hidden[k], res["r"])
+    return wl.K * rows
+
+
+def prepare_oracle_sample(wl, rows: int):
+    import oracle.solo_oracle as orc
+    dec = orc.bf16_bits_to_f64
+    hidden = [dec(synth.gen_hidden(wl, k, 0, rows)) for k in range(wl.K)]
+    W = dec(synth.gen_W(wl))
+    gamma = dec(synth.gen_gamma(wl))
+    targets = synth.gen_targets(wl)[:, :rows]
+    return hidden, gamma, W, targets
+
+
+def blas_threads() -> int:
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def cpu_baseline(wl, seconds: float):
+    probe = 16
+    data = prepare_oracle_sample(wl, 4096)
+    sub = lambda n: ([h[:n] for h in data[0]], data[1], data[2], data[3][:, :n])
+    oracle_sample(wl, probe, sub(probe))
+    t = time.perf_counter()
+    oracle_sample(wl, probe, sub(probe))
+    per_row = (time.perf_counter() - t) / probe
+    rows = int(min(4096, max(probe, seconds / max(per_row, 1e-9))))
+    t = time.perf_counter()
+    toks = oracle_sample(wl, rows, sub(rows))
+    dt = time.perf_counter() - t
+    return {"value": toks / dt, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+            "sample": f"first {rows} tokens of each of the {wl.K} modules (full V={wl.V}, "
+                      f"d={wl.d}), forward + dH, dW/dgamma terms of the final module's "
+                      f"sample; fp64 numpy oracle, {dt:.1f} s"}
+
+
+def run_reference(args, wl):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    rows = 32
+    data = prepare_oracle_sample(wl, rows)
+    for _ in range(args.warmup):
+        oracle_sample(wl, rows, data)
+    t = time.perf_counter()
+    toks = 0
+    for _ in range(args.steps):
+        toks += oracle_sample(wl, rows, data)
+    dt = time.perf_counter() - t
+    value = toks / dt
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "K": wl.K, "N": wl.N, "d": wl.d, "V": wl.V,
+                       "parallelism": "rank 0 only"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": blas_threads(),
+                             "kind": "oracle",
+                             "sample": f"each step: first {rows} tokens of each of the {wl.K} "
+                                       f"modules at full V and d"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------- GPU leg
+
+def run_ours(args, wl):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_35440_gb300 import solo_readout as sr
+    from paper_2609_35440_gb300 import build
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else torch.cuda.current_device())
+
+    build.ensure_built()
+    sr.load()
+    stream = torch.cuda.current_stream(dev)
+
+    # inputs resident in HBM (seeded; ranks use distinct seeds: independent replicas)
+    wlr = wl.with_(seed=wl.seed + 1000 * rank) if rank else wl
+    inp = synth.generate(wlr)
+    to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    hidden = [to_dev(inp.hidden[k]) for k in range(wl.K)]
+    gamma, W = to_dev(inp.gamma), to_dev(inp.W)
+    targets = torch.from_numpy(inp.targets).to(dev)
+    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index, device=dev)
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    clk = ClockSampler(dev.index).__enter__()
+    time.sleep(1.0)                      # let the sampler start before the warm-up
+    for _ in range(max(args.warmup, 0)):
+        ro(hidden, gamma, W, targets, stream=stream)
+    barrier()
+
+    # ---- device-resident timing of exactly `steps` calls; events recorded on the
+    # launching stream between the stages of every call (read after the loop)
+    step_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(sr.SOLO_NUM_STAGES + 1)]
+                for _ in range(args.steps)]
+    for evl in step_evs:
+        for e in evl:
+            e.record(stream)
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    t0.record(stream)
+    for i in range(args.steps):
+        ro(hidden, gamma, W, targets, stream=stream, events=step_evs[i])
+    t1.record(stream)
+    barrier()
+    clk.__exit__(None, None, None)
+    flags = ro.flags(stream)
+    ms = t0.elapsed_time(t1)
+    stage_ms = np.zeros(sr.SOLO_NUM_STAGES)
+    for evl in step_evs:
+        stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(sr.SOLO_NUM_STAGES)]
+    stage_ms /= args.steps
+
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+
+    tokens_step = wl.M
+    value = world * tokens_step * args.steps / (ms / 1e3)
+
+    # ---- end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        h_host = [torch.from_numpy(np.ascontiguousarray(inp.hidden[k]).view(np.int16)).view(
+            torch.bfloat16).pin_memory() for k in range(wl.K)]
+        t_host = torch.from_numpy(inp.targets).pin_memory()
+        lt_host = torch.empty(wl.K, wl.N, dtype=torch.float32).pin_memory()
+        lm_host = torch.empty(wl.K, dtype=torch.float32).pin_memory()
+        steps_e2e = max(3, min(args.steps, 10))
+
+        def e2e_step():
+            for k in range(wl.K):
+                hidden[k].copy_(h_host[k], non_blocking=True)
+            targets.copy_(t_host, non_blocking=True)
+            ro(hidden, gamma, W, targets, stream=stream)
+            lt_host.copy_(ro.loss_tok, non_blocking=True)
+            lm_host.copy_(ro.loss_mean, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        barrier()
+        t0.record(stream)
+        for _ in range(steps_e2e):
+            e2e_step()
+        t1.record(stream)
+        barrier()
+        ems = t0.elapsed_time(t1)
+        if world > 1:
+            tt = torch.tensor([ems], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ems = float(tt.item())
+        h2d = sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4
+        d2h = lt_host.numel() * 4 + lm_host.numel() * 4
+        e2e = {"value": world * tokens_step * steps_e2e / (ems / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    peaks, peak_src = load_peaks()
+    G = costmodel.gemm_flops(wl.M, wl.V, wl.d)     # one module-GEMM over all K modules
+    names = sr.STAGE_NAMES
+    gemm_stage_flops = {"logits": G, "dxhat": G, "dW": G / wl.K}
+    dom = max(gemm_stage_flops, key=lambda s: stage_ms[names.index(s)])
+    dom_ms = stage_ms[names.index(dom)]
+    achieved = gemm_stage_flops[dom] / (dom_ms / 1e3) / 1e12
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    traffic = committed_traffic(wl) if dom == "logits" else None
+    algo = costmodel.call_flops(wl.K, wl.N, wl.d, wl.V)
+    step_s = ms / 1e3 / args.steps
+    cpu = None
+    if not args.no_cpu:
+        cpu = cpu_baseline(wl, args.cpu_seconds)
+    # rmsnorm, logits, lse + module means, grad, dxhat, norm_bwd, dgamma parts, dW, dgamma
+    launches_per_step = 10
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "K": wl.K, "N": wl.N, "d": wl.d, "V": wl.V,
+                   "global_batch_tokens": world * wl.M, "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (hidden+W 265 MB; 2.1 GB gradient buffer "
+                         "written per step)"},
+        "algo_tflops": algo / step_s / 1e12,
+        "algo_frac_of_peak": algo / step_s / 1e12 / peak,
+        "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
+        "roofline": {"bound": "tensor", "kernel": f"{dom} GEMM (tcgen05)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside "
+                                    f"back-to-back steps)"},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "clocks": clk.summary(),
+        "gpu_launches": launches_per_step * args.steps,
+        "device_flags": flags,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    wl = workload_from_name(args.workload)
+    if args.warmup < 0 or args.steps < 1:
+        raise SystemExit("need --steps >= 1")
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    main()

@@ -39,6 +39,29 @@ __device__ __forceinline__ bool token_kept(const RowArgs& a, int64_t row, int y)
 }
 
 // ---- final RMSNorm: r_i = (mean_j h_ij^2 + eps)^-1/2, xhat = bf16(gamma h r) ------
+// The bf16 rounding of xhat is a quantisation decision, so it is taken on the
+// exact value: the sum of squares is accumulated error-free (each h^2 of a
+// bf16 h is exact in fp32; TwoSum keeps the rounding error of every add),
+// r is formed in fp64, and a product whose fp32 value lies within a few ulp
+// of a bf16 rounding midpoint is decided against the midpoint in fp64.
+
+__device__ __forceinline__ uint16_t xhat_bf16(float gh, float r32, double r64) {
+  const float y = gh * r32;           // gh = gamma * h is exact in fp32
+  const uint32_t b = __float_as_uint(y);
+  const uint32_t mag = b & 0x7FFFFFFFu;
+  const int low = static_cast<int>(mag & 0xFFFFu) - 0x8000;
+  if (low >= -4 && low <= 4 && mag < 0x7F000000u && mag >= 0x00800000u) {
+    // |y32 - y| <= 2 ulp, so the exact value lies strictly between the two
+    // neighbouring bf16 values; compare it with their midpoint.
+    const uint32_t down = mag & 0xFFFF0000u;
+    const double mid = static_cast<double>(__uint_as_float(down | 0x8000u));
+    const double ya = fabs(static_cast<double>(gh) * r64);
+    uint32_t q = down >> 16;
+    if (ya > mid || (ya == mid && (q & 1u))) q += 1;
+    return static_cast<uint16_t>(q | ((b >> 16) & 0x8000u));
+  }
+  return static_cast<uint16_t>((b + 0x7FFFu + ((b >> 16) & 1u)) >> 16);
+}
 
 __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
@@ -50,27 +73,37 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
   const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
   const int nv = a.d / 8;
-  float ss = 0.f;
+  float s = 0.f, c = 0.f;
   for (int v = lane; v < nv; v += 32) {
     float f[8];
     unpack8(__ldg(h + v), f);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) ss = fmaf(f[j], f[j], ss);
+    for (int j = 0; j < 8; ++j) {
+      const float x = f[j] * f[j];
+      const float t = s + x;
+      const float bb = t - s;
+      c += (s - (t - bb)) + (x - bb);
+      s = t;
+    }
   }
-  ss = warp_sum(ss);
-  const float r = 1.0f / sqrtf(ss / static_cast<float>(a.d) + a.eps);
+  double ss = static_cast<double>(s) + static_cast<double>(c);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const double r64 = 1.0 / sqrt(ss / static_cast<double>(a.d) + static_cast<double>(a.eps));
+  const float r = static_cast<float>(r64);
   uint4* out = reinterpret_cast<uint4*>(a.xhat + row * a.d);
   for (int v = lane; v < nv; v += 32) {
     float f[8], gg[8];
     unpack8(__ldg(h + v), f);
     unpack8(__ldg(g + v), gg);
-    uint4 o;
-    // gamma * h is exact in fp32 (8 x 8 significant bits); one rounding for * r.
-    o.x = pack2(gg[0] * f[0] * r, gg[1] * f[1] * r);
-    o.y = pack2(gg[2] * f[2] * r, gg[3] * f[3] * r);
-    o.z = pack2(gg[4] * f[4] * r, gg[5] * f[5] * r);
-    o.w = pack2(gg[6] * f[6] * r, gg[7] * f[7] * r);
-    out[v] = o;
+    uint32_t w[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t lo = xhat_bf16(gg[2 * j] * f[2 * j], r, r64);
+      const uint32_t hi = xhat_bf16(gg[2 * j + 1] * f[2 * j + 1], r, r64);
+      w[j] = lo | (hi << 16);
+    }
+    out[v] = make_uint4(w[0], w[1], w[2], w[3]);
   }
   if (lane == 0) a.r[row] = r;
 }

@@ -65,9 +65,10 @@ def oracle_full(wl, inp: synth.Inputs, mask=None, targets=None):
     dec = orc.bf16_bits_to_f64
     hidden = [dec(inp.hidden[k]) for k in range(wl.K)]
     tg = inp.targets if targets is None else targets
+    # the library receives eps as fp32; the oracle uses that same value
     return orc.solo_readout_fwd_bwd(hidden, dec(inp.gamma), dec(inp.W), tg.astype(np.int64),
-                                    mask, eps=wl.eps, ignore_index=wl.ignore_index,
-                                    contract=True)
+                                    mask, eps=float(np.float32(wl.eps)),
+                                    ignore_index=wl.ignore_index, contract=True)
 
 
 def max_rel(a, ref) -> float:
@@ -116,4 +117,59 @@ def compare_full(wl, gpu, ref, check_dW=True, check_dgamma=True):
         check_grad("dW", gpu["dW"], ref["dW"], rep)
     if check_dgamma:
         check_grad("dgamma", gpu["dgamma"], ref["dgamma"], rep)
+    return rep
+
+
+def sampled_check(wl, inp: synth.Inputs, gpu, rows_per_module=24, n_vocab=48, seed=0,
+                  full_final=True, chunk=512):
+    """Parity at full size on sampled outputs the oracle computes one by one.
+
+    For every module: the first and last token and random tokens: token loss
+    (abs err) and dH rows (max rel err and cosine over the sampled rows).  The
+    module mean must equal the mean of the kept token losses (a property).
+    With ``full_final`` the final module is run through the oracle in chunks:
+    its mean loss, every dgamma entry and the dW rows of sampled vocabulary
+    entries (including heavy rows and frequent targets) are compared.
+    """
+    rng = np.random.default_rng(seed)
+    dec = orc.bf16_bits_to_f64
+    gamma, W = dec(inp.gamma), dec(inp.W)
+    eps = float(np.float32(wl.eps))
+    rep = {}
+    for k in range(wl.K):
+        y = inp.targets[k].astype(np.int64)
+        kept, _ = orc.kept_tokens(y, None, wl.V, wl.ignore_index)
+        nv = int(kept.sum())
+        rows = np.unique(np.concatenate([[0, wl.N - 1],
+                                         rng.choice(wl.N, min(rows_per_module, wl.N), replace=False)]))
+        res = orc.module_rows(dec(inp.hidden[k][rows]), gamma, W, y[rows], kept[rows], nv, eps, True)
+        err = float(np.max(np.abs(gpu["loss_tok"][k][rows] - res["loss"])))
+        rep[f"loss_tok[{k}]"] = err
+        assert err <= LOSS_TOK_ABS, ("loss_tok", k, err)
+        check_grad(f"dH[{k}] rows", gpu["dhidden"][k][rows], res["dh"], rep)
+        mean_prop = float(np.sum(gpu["loss_tok"][k][kept], dtype=np.float64) / max(nv, 1))
+        assert abs(gpu["loss_mean"][k] - mean_prop) <= 1e-6 * max(1.0, abs(mean_prop)), \
+            ("loss_mean property", k, gpu["loss_mean"][k], mean_prop)
+    if full_final:
+        k = wl.K - 1
+        y = inp.targets[k].astype(np.int64)
+        kept, _ = orc.kept_tokens(y, None, wl.V, wl.ignore_index)
+        Wrms = np.sqrt(np.mean(W * W, axis=1))
+        heavy = np.nonzero(Wrms > 5 * np.median(Wrms))[0][:8]
+        freq = np.argsort(-np.bincount(y[kept], minlength=wl.V))[:8]
+        cols = np.unique(np.concatenate([[0, wl.V - 1], heavy, freq,
+                                         rng.choice(wl.V, n_vocab, replace=False)]))
+        ch = orc.final_module_chunked(lambda i0, n: dec(inp.hidden[k][i0:i0 + n]), wl.N, gamma,
+                                      W, y, kept, eps, True, dW_cols=cols, chunk=chunk)
+        want = ch["loss"].sum() / max(ch["n_valid"], 1)
+        rel = abs(gpu["loss_mean"][k] - want) / abs(want)
+        rep["loss_mean_final_rel"] = rel
+        assert rel <= LOSS_MEAN_REL, ("loss_mean", k, gpu["loss_mean"][k], want)
+        check_grad("dgamma", gpu["dgamma"], ch["dgamma"], rep)
+        check_grad("dW rows", gpu["dW"][cols], ch["dW_rows"], rep)
+    # each column of dW sums to zero over the vocabulary (rows of G sum to zero)
+    colsum = np.abs(gpu["dW"].sum(axis=0))
+    scale = np.sqrt(np.sum(gpu["dW"] ** 2, axis=0)) + 1e-30
+    rep["dW_colsum_rel"] = float(np.max(colsum / scale))
+    assert rep["dW_colsum_rel"] < 1e-2, rep["dW_colsum_rel"]
     return rep
