@@ -53,7 +53,9 @@ enum {
   SOLO_ERR_WORKSPACE_TOO_SMALL = -3, /* workspace_bytes below the query result */
   SOLO_ERR_CUDA = -4,                /* a CUDA runtime call failed */
   SOLO_ERR_NOT_SM103 = -5,           /* current device is not compute capability 10.3 */
-  SOLO_ERR_MISALIGNED = -6           /* a tensor pointer is not 16-byte aligned */
+  SOLO_ERR_MISALIGNED = -6,          /* a tensor pointer is not 16-byte aligned */
+  SOLO_ERR_EXCEEDS_STATIC_SCRATCH = -7 /* solo_readout_fwd_bwd_static: the problem needs
+                                          more than SOLO_STATIC_SCRATCH_BYTES of scratch */
 };
 
 /* Device-detected conditions, OR-ed into the workspace flag word. */
@@ -173,6 +175,54 @@ const char* solo_readout_strerror(solo_status_t status);
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 int32_t solo_readout_version(void);
+
+/*
+ * Size of the library's built-in scratch area used by
+ * solo_readout_fwd_bwd_static: 64 MiB of device memory, reserved on every GPU
+ * that loads the library's device code and held until the process exits.
+ */
+#define SOLO_STATIC_SCRATCH_BYTES (64u << 20)
+
+/*
+ * The same forward + backward as solo_readout_fwd_bwd, for callers that
+ * cannot allocate device memory and so cannot supply a workspace: code that
+ * runs where allocation is forbidden or unavailable, such as an inference or
+ * plugin host that lets a step enqueue work but never allocate, or a loop
+ * that froze its memory use after start-up.  This paper has no counterpart
+ * of it; it is an addition of this library.
+ *
+ * Instead of a caller workspace it uses a fixed scratch array compiled into
+ * the library (SOLO_STATIC_SCRATCH_BYTES).  The call itself allocates
+ * nothing.  Limits and rules:
+ *  - Problems whose solo_readout_workspace_bytes exceeds
+ *    SOLO_STATIC_SCRATCH_BYTES are rejected with
+ *    SOLO_ERR_EXCEEDS_STATIC_SCRATCH before anything is enqueued (roughly
+ *    K*N*(2V + 6d + 48) bytes must fit; e.g. K=2, N=256, d=128, V=4096 uses
+ *    about 6 MiB).
+ *  - The first call on a device looks up the device address of the scratch
+ *    array for that device (the array's name in host code is not a device
+ *    address).  Make that first call before any stream capture.
+ *  - Every call on a device shares the one array, and it keeps the previous
+ *    call's contents; the call clears what must start at zero itself.  Calls
+ *    whose execution overlaps on the GPU (other streams, other host
+ *    threads) race on the scratch and give wrong results: serialise them.
+ *  - device_flags: NULL, or a device uint32 that receives this call's flag
+ *    word (SOLO_FLAG_*) at the end of the call, asynchronously on `stream`.
+ * Every other argument means what it means for solo_readout_fwd_bwd.
+ */
+solo_status_t solo_readout_fwd_bwd_static(const solo_dims_t* dims,
+                                          const solo_bf16_t* const* hidden,
+                                          const solo_bf16_t* gamma,
+                                          const solo_bf16_t* W,
+                                          const int32_t* targets,
+                                          const uint8_t* mask,
+                                          float* loss_tok,
+                                          float* loss_mean,
+                                          solo_bf16_t* const* dhidden,
+                                          float* dW,
+                                          float* dgamma,
+                                          uint32_t* device_flags,
+                                          solo_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -359,6 +359,9 @@ const char* solo_readout_strerror(solo_status_t status) {
     case SOLO_ERR_CUDA: return "a CUDA runtime call failed";
     case SOLO_ERR_NOT_SM103: return "current device is not compute capability 10.3 (sm_103a)";
     case SOLO_ERR_MISALIGNED: return "a tensor pointer is not suitably aligned (16 bytes)";
+    case SOLO_ERR_EXCEEDS_STATIC_SCRATCH:
+      return "problem needs more scratch than the 64 MiB built-in array of "
+             "solo_readout_fwd_bwd_static; use solo_readout_fwd_bwd with a workspace";
     default: return "unknown status";
   }
 }
@@ -366,3 +369,61 @@ const char* solo_readout_strerror(solo_status_t status) {
 int32_t solo_readout_version(void) { return 100; }
 
 }  // extern "C"
+
+// ---- allocation-free variant -----------------------------------------------------
+// For callers that cannot allocate device memory.  The scratch that
+// solo_readout_fwd_bwd takes from the caller's workspace comes instead from a
+// fixed array compiled into this file's device code.  In host code the name
+// g_static_scratch is only a host-side stand-in for the symbol, so its device
+// address is looked up per device with cudaGetSymbolAddress (on the first call
+// on that device) and that address is what the kernels receive.
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_static_scratch[SOLO_STATIC_SCRATCH_BYTES];
+
+std::mutex g_static_mu;
+void* g_static_ptr[64] = {};
+
+// Device address of the scratch array on the current device, looked up once.
+solo_status_t static_scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return SOLO_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr)
+      return SOLO_ERR_CUDA;
+    g_static_ptr[dev] = p;
+  }
+  *out = g_static_ptr[dev];
+  return SOLO_OK;
+}
+
+}  // namespace
+
+extern "C" solo_status_t solo_readout_fwd_bwd_static(
+    const solo_dims_t* dims, const solo_bf16_t* const* hidden, const solo_bf16_t* gamma,
+    const solo_bf16_t* W, const int32_t* targets, const uint8_t* mask, float* loss_tok,
+    float* loss_mean, solo_bf16_t* const* dhidden, float* dW, float* dgamma,
+    uint32_t* device_flags, solo_stream_t stream) {
+  size_t need = 0;
+  solo_status_t st = solo_readout_workspace_bytes(dims, &need);
+  if (st != SOLO_OK) return st;
+  if (need > SOLO_STATIC_SCRATCH_BYTES) return SOLO_ERR_EXCEEDS_STATIC_SCRATCH;
+  if (device_flags && (reinterpret_cast<uintptr_t>(device_flags) & 3u)) return SOLO_ERR_MISALIGNED;
+  void* scratch = nullptr;
+  st = static_scratch_address(&scratch);
+  if (st != SOLO_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // The launch sequence clears the flag word itself; every other scratch
+  // buffer is written before it is read, so stale contents never leak.
+  st = run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
+           scratch, SOLO_STATIC_SCRATCH_BYTES, s, nullptr, 0);
+  if (st != SOLO_OK) return st;
+  if (device_flags &&
+      cudaMemcpyAsync(device_flags, scratch, sizeof(uint32_t), cudaMemcpyDeviceToDevice, s) !=
+          cudaSuccess)
+    return SOLO_ERR_CUDA;
+  return SOLO_OK;
+}

@@ -21,6 +21,8 @@ SOLO_ERR_WORKSPACE_TOO_SMALL = -3
 SOLO_ERR_CUDA = -4
 SOLO_ERR_NOT_SM103 = -5
 SOLO_ERR_MISALIGNED = -6
+SOLO_ERR_EXCEEDS_STATIC_SCRATCH = -7
+SOLO_STATIC_SCRATCH_BYTES = 64 << 20
 
 SOLO_FLAG_BAD_TARGET = 1
 SOLO_FLAG_TIMEOUT = 2
@@ -72,6 +74,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_get_flags.restype = i32
     lib.solo_readout_strerror.argtypes = [i32]
     lib.solo_readout_strerror.restype = ctypes.c_char_p
+    lib.solo_readout_fwd_bwd_static.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp, vp,
+                                                 vp, ctypes.POINTER(vp), vp, vp, vp, vp]
+    lib.solo_readout_fwd_bwd_static.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
     _lib = lib
@@ -151,6 +156,25 @@ def solo_readout_fwd_bwd_events(dims, hidden, gamma, W, targets, mask, loss_tok,
                extra=(arr, len(handles)))
     if check and st != SOLO_OK:
         raise SoloError(st, "solo_readout_fwd_bwd_events")
+    return st
+
+
+def solo_readout_fwd_bwd_static(dims: solo_dims_t, hidden: Sequence, gamma, W, targets, mask,
+                                loss_tok, loss_mean, dhidden: Sequence, dW, dgamma,
+                                device_flags=None, stream=None, check: bool = True) -> int:
+    """The allocation-free variant: the library's built-in scratch replaces the
+    workspace (problems up to SOLO_STATIC_SCRATCH_BYTES of scratch)."""
+    K = dims.K
+    if len(hidden) != K or len(dhidden) != K:
+        raise ValueError("hidden and dhidden need K entries")
+    harr = (ctypes.c_void_p * K)(*[_ptr(h) for h in hidden])
+    darr = (ctypes.c_void_p * K)(*[_ptr(h) for h in dhidden])
+    st = load().solo_readout_fwd_bwd_static(
+        ctypes.byref(dims), harr, _ptr(gamma), _ptr(W), _ptr(targets), _ptr(mask),
+        _ptr(loss_tok), _ptr(loss_mean), darr, _ptr(dW), _ptr(dgamma), _ptr(device_flags),
+        _stream_handle(stream))
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd_static")
     return st
 
 
