@@ -1,19 +1,29 @@
-// Persistent tcgen05 GEMM for sm_103a with three fused epilogues.
+// Persistent tcgen05 GEMM for sm_103a on CTA pairs, with three fused epilogues.
 //
-// One CTA per SM loops over 128 x 256 output tiles.  Warp 0 streams 64-wide
-// reduction blocks of A and B into a 4-stage shared-memory ring with TMA
-// (128-byte swizzle), warp 1 issues tcgen05.mma (M=128, N=256, K=16, bf16 in,
-// fp32 accumulate) into one of two TMEM accumulators of 256 columns, and
-// warps 2-5 drain the other accumulator (each warp owns 32 TMEM lanes = 32
-// rows of the tile) while the next tile is being multiplied.
+// Two CTAs on neighbouring SMs form a cluster and compute one 256 x 256
+// output tile together with tcgen05.mma.cta_group::2 (M = 256, N = 256, K =
+// 16, bf16 in, fp32 accumulate).  Each CTA stages its own 128 rows of A and
+// its own 128 columns of B per 64-wide reduction block (32 KB), so a 6-stage
+// ring fits in shared memory and each SM needs 64 B of operands per clock at
+// full MMA rate (a single-CTA 128 x 256 tile needs 96 B and only has room
+// for 4 stages).  Roles, in both CTAs:
+//   warp 0     TMA producer: loads its CTA's A and B halves, completion is
+//              signalled on the even CTA's "full" barrier (pair-mode TMA)
+//   warp 1     even CTA: one thread issues the pair MMAs into one of two TMEM
+//              accumulators of 256 columns and commits (multicast) to both
+//              CTAs' "empty" and "tmem full" barriers; both CTAs' warp 1
+//              allocate / free the tensor memory together
+//   warps 2-5  epilogue: each owns 32 TMEM lanes (rows) of its CTA's 128
+//              rows x 256 columns; releases the accumulator on the even CTA's
+//              "tmem empty" barrier (8 arrivals: 4 warps x 2 CTAs)
 //
 // Epilogues:
-//  kLogits  Z = Xhat W^T.  Per row and tile: m = max_v z, s = sum_v exp(z - m),
-//           the target logit when the target falls in the tile, and the bf16
-//           values exp(z - m) written to a [rows, V] buffer with TMA stores.
-//           These feed the log-sum-exp of the cross-entropy (Eq. 2 and the
-//           local loss of Algorithm 1) and, rescaled, its gradient, so the
-//           logits are never written and never recomputed.
+//  kLogits  Z = Xhat W^T.  Per row and 256-column tile: m = max_v z,
+//           s = sum_v exp(z - m), the target logit when the target falls in the
+//           tile, and the bf16 values exp(z - m) written to a [rows, V] buffer
+//           with TMA stores.  These feed the log-sum-exp of the cross-entropy
+//           (Eq. 2 and the local loss of Algorithm 1) and, rescaled, its
+//           gradient, so the logits are never written and never recomputed.
 //  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3; fp32 out.
 //  kDW      dW = G^T Xhat over the final module's tokens; fp32 out.
 //
@@ -26,9 +36,11 @@
 namespace solo {
 namespace {
 
+constexpr int kPairRows = 2 * kBM;                  // 256 output rows per CTA pair
+constexpr int kBHalf = kBN / 2;                     // B columns staged per CTA
 constexpr int kABytes = kBM * kBK * 2;              // 16 KB
-constexpr int kBBytes = kBN * kBK * 2;              // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBBytes = kBHalf * kBK * 2;           // 16 KB
+constexpr int kStageBytes = kABytes + kBBytes;      // per CTA
 constexpr int kEpiBufBytes = 32 * 128;              // 32 rows x 128 B
 constexpr int kEpiWarps = 4;
 constexpr int kTmemCols = 2 * kBN;                  // two accumulators
@@ -39,8 +51,11 @@ constexpr int kSmemBar = kSmemEpi + kEpiWarps * 2 * kEpiBufBytes;
 constexpr int kNumBars = 2 * kStages + 2 + 2 + 1;
 constexpr int kSmemMisc = kSmemBar + kNumBars * 8;
 constexpr int kSmemTotal = kSmemMisc + 16 + 1024;   // + alignment slack
+static_assert(kSmemTotal <= 232448, "shared memory budget");
 
 constexpr float kLog2e = 1.4426950408889634f;
+
+constexpr uint16_t kBothCtas = 0x3;
 
 __device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, int& nb) {
   const int per_group = a.group_m * a.n_blocks;
@@ -57,18 +72,23 @@ __device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, i
 __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
   const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait(a, parity)) {
+  while (!mbar_try_wait_cluster(a, parity)) {
     if (globaltimer_ns() - t0 > kWaitLimitNs) break;
   }
 }
 
+__device__ __forceinline__ void spin_ns(uint64_t ns) {
+  const uint64_t t0 = globaltimer_ns();
+  while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
+}
+
 template <int MODE>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmD, const GemmArgs args) {
   constexpr bool kAmn = (MODE == kDW);
   constexpr bool kBmn = (MODE != kLogits);
-  constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN, kAmn, kBmn);
+  constexpr uint32_t kIdesc = idesc_bf16_f32(kPairRows, kBN, kAmn, kBmn);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -84,6 +104,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();       // 0: even CTA (issues the MMAs), 1: odd
+  const bool even = rank == 0;
+  const int cluster = blockIdx.x >> 1;
+  const int num_clusters = gridDim.x >> 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -92,7 +116,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], kEpiWarps);
+      mbar_init(&tempty[a], 2 * kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -102,46 +126,50 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tma_prefetch_desc(&tmD);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();            // the peer's barriers exist before anything signals them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
+      const uint32_t full_even = map_to_rank(smem_u32(full), 0);
       uint32_t stage = 0, phase = 0;
       uint32_t issued = 0, last_phase = 0;   // per-stage bits for draining
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < args.num_tiles; t += gridDim.x) {
+      for (int t = cluster; ok && t < args.num_tiles; t += num_clusters) {
         int mb, nb;
         tile_coords(t, args, mb, nb);
-        const int m0 = mb * kBM, n0 = nb * kBN;
+        const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
+        const int n0 = nb * kBN + static_cast<int>(rank) * kBHalf;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+          if (!mbar_wait_cluster(&empty[stage], phase ^ 1, abort_flag)) {
             ok = false;
             break;
           }
           uint8_t* sA = smem + kSmemA + stage * kABytes;
           uint8_t* sB = smem + kSmemB + stage * kBBytes;
-          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          if (even) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
+          const uint32_t fb = full_even + stage * 8;
           const int kr = args.k_row0 + kb * kBK;
           if constexpr (!kAmn) {
-            tma_load_2d(sA, &tmA, &full[stage], kb * kBK, m0);
+            tma_load_2d_pair(sA, &tmA, fb, kb * kBK, m0);
           } else {
 #pragma unroll
             for (int c = 0; c < kBM / 64; ++c)
-              tma_load_2d(sA + c * 8192, &tmA, &full[stage], m0 + 64 * c, kr);
+              tma_load_2d_pair(sA + c * 8192, &tmA, fb, m0 + 64 * c, kr);
           }
           if constexpr (!kBmn) {
-            tma_load_2d(sB, &tmB, &full[stage], kb * kBK, n0);
+            tma_load_2d_pair(sB, &tmB, fb, kb * kBK, n0);
           } else {
 #pragma unroll
-            for (int c = 0; c < kBN / 64; ++c)
-              tma_load_2d(sB + c * 8192, &tmB, &full[stage], n0 + 64 * c, kr);
+            for (int c = 0; c < kBHalf / 64; ++c)
+              tma_load_2d_pair(sB + c * 8192, &tmB, fb, n0 + 64 * c, kr);
           }
           issued |= 1u << stage;
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
@@ -152,10 +180,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
       }
       if (ok) {
-        // Tail: wait until the MMA warp has released every stage, so that no
-        // tcgen05.commit arrival is still pending when the CTA exits.
+        // Tail: wait until the MMAs have released every stage, so that no
+        // commit arrival is still pending when the CTA exits.
         for (int i = 0; ok && i < kStages; ++i) {
-          ok = mbar_wait(&empty[stage], phase ^ 1, abort_flag);
+          ok = mbar_wait_cluster(&empty[stage], phase ^ 1, abort_flag);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1;
@@ -164,30 +192,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       if (!ok) {
         atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
-        for (int s = 0; s < kStages; ++s)
-          if (issued & (1u << s)) mbar_drain(&full[s], (last_phase >> s) & 1u);
+        if (even) {
+          // the even CTA's full barriers count both CTAs' bytes
+          for (int s = 0; s < kStages; ++s)
+            if (issued & (1u << s)) mbar_drain(&full[s], (last_phase >> s) & 1u);
+        } else {
+          spin_ns(200000);   // let this CTA's in-flight loads land
+        }
       }
     }
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    if (even && lane == 0) {
       uint32_t stage = 0, phase = 0;
       int local = 0;
       bool ok = true;
       const uint32_t a_base = smem_u32(smem + kSmemA);
       const uint32_t b_base = smem_u32(smem + kSmemB);
-      for (int t = blockIdx.x; ok && t < args.num_tiles; t += gridDim.x, ++local) {
+      for (int t = cluster; ok && t < args.num_tiles; t += num_clusters, ++local) {
         const uint32_t acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag)) {
+        if (!mbar_wait_cluster(&tempty[acc], acc_phase ^ 1, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * kBN;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag)) {
+          if (!mbar_wait_cluster(&full[stage], phase, abort_flag)) {
             ok = false;
             break;
           }
@@ -200,20 +233,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                      : smem_desc_sw128(sa + k * 32, 16, 1024);
             const uint64_t bd = kBmn ? smem_desc_sw128(sb + k * 2048, 8192, 1024)
                                      : smem_desc_sw128(sb + k * 32, 16, 1024);
-            mma_bf16(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+            mma_bf16_pair(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
           }
-          mma_commit(&empty[stage]);
+          mma_commit_pair(&empty[stage], kBothCtas);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1;
           }
         }
         if (!ok) break;
-        mma_commit(&tfull[acc]);
+        mma_commit_pair(&tfull[acc], kBothCtas);
       }
       if (!ok) {
         atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
-        mma_commit(drain);
+        mma_commit_pair(drain, 0x1);
         mbar_drain(drain, 0);
       }
     }
@@ -223,16 +256,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int q = warp & 3;                  // TMEM lane quadrant = row block of 32
     const int ew = warp - 2;                 // staging buffer owner
     uint8_t* ebuf = smem + kSmemEpi + ew * 2 * kEpiBufBytes;
+    const uint32_t tempty_even = map_to_rank(smem_u32(tempty), 0);
     int buf = 0;
     int local = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < args.num_tiles; t += gridDim.x, ++local) {
+    for (int t = cluster; t < args.num_tiles; t += num_clusters, ++local) {
       int mb, nb;
       tile_coords(t, args, mb, nb);
-      const int m0 = mb * kBM, n0 = nb * kBN;
+      const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
+      const int n0 = nb * kBN;
       const uint32_t acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(&tfull[acc], acc_phase, abort_flag));
+      ok = __all_sync(0xffffffffu, mbar_wait_cluster(&tfull[acc], acc_phase, abort_flag));
       if (!ok) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(32 * q) << 16) + acc * kBN;
@@ -249,13 +284,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           if (c * 32 >= ncols) break;
           float v[32];
           tmem_ld32(tbase + c * 32, v);
+          const int yc = has_y ? yrel - c * 32 : -1;   // target column within this chunk
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
+          for (int j = 0; j < 32; ++j) {
             if (c * 32 + j < ncols) mx = fmaxf(mx, v[j]);
-          if (has_y && (yrel >> 5) == c) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (j == (yrel & 31)) zyv = v[j];
+            zyv = (j == yc) ? v[j] : zyv;
           }
         }
         const float mlog = mx * kLog2e;
@@ -301,7 +334,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[acc]);
+        if (lane == 0) {
+          if (even) mbar_arrive(&tempty[acc]);
+          else mbar_arrive_remote(tempty_even + acc * 8);
+        }
         if (row_ok) args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
         if (has_y) args.zy[row] = zyv;
       } else {
@@ -329,7 +365,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[acc]);
+        if (lane == 0) {
+          if (even) mbar_arrive(&tempty[acc]);
+          else mbar_arrive_remote(tempty_even + acc * 8);
+        }
       }
     }
     if (!ok && lane == 0) atomicOr(args.flags, SOLO_FLAG_TIMEOUT);
@@ -339,9 +378,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  cluster_sync();            // no CTA leaves while its peer may still signal it
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
@@ -363,9 +403,11 @@ cudaError_t gemm_prepare(int /*device*/) {
 }
 
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
-                        const CUtensorMap& d, const GemmArgs& args, int grid,
+                        const CUtensorMap& d, const GemmArgs& args, int sms,
                         cudaStream_t stream) {
   if (args.num_tiles <= 0) return cudaSuccess;
+  const int clusters = std::min(args.num_tiles, std::max(sms / 2, 1));
+  const int grid = 2 * clusters;
   switch (mode) {
     case kLogits:
       gemm_kernel<kLogits><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);

@@ -7,11 +7,12 @@
 
 namespace solo {
 
-// Tensor-core tile: 128 rows x 256 columns per CTA, reduction in blocks of 64.
+// Tensor-core tile: a CTA pair computes 256 rows x 256 columns (each CTA owns
+// 128 rows), reduction in blocks of 64 through a 6-stage shared-memory ring.
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
-constexpr int kStages = 4;
+constexpr int kStages = 6;
 constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
 // The three products of one call.
@@ -28,8 +29,8 @@ struct GemmArgs {
   int32_t N;          // columns of the product
   int32_t k_blocks;   // reduction length / kBK, rounded up
   int32_t k_row0;     // first reduction row in A/B coordinates (kDW: first token of the module)
-  int32_t m_blocks;
-  int32_t n_blocks;
+  int32_t m_blocks;   // 256-row blocks (one per CTA pair)
+  int32_t n_blocks;   // 256-column blocks
   int32_t group_m;    // tile raster: group_m row blocks sweep all column blocks together
   int32_t num_tiles;
   // kLogits epilogue
@@ -42,8 +43,9 @@ struct GemmArgs {
 
 size_t gemm_smem_bytes();
 cudaError_t gemm_prepare(int device);  // sets the dynamic shared memory limit once per device
+// Launches min(tiles, sms / 2) CTA pairs.
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
-                        const CUtensorMap& d, const GemmArgs& args, int grid,
+                        const CUtensorMap& d, const GemmArgs& args, int sms,
                         cudaStream_t stream);
 
 // ---- row kernels ---------------------------------------------------------------

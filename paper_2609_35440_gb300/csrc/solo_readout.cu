@@ -26,7 +26,10 @@ using namespace solo;
 
 constexpr size_t kAlign = 1024;
 constexpr int kDgRows = 64;
-constexpr int kGroupM = 16;
+// Tile raster (in 256-row pair blocks) per product, from a sweep on GB300.
+constexpr int kGroupLogits = 16;
+constexpr int kGroupDxhat = 4;
+constexpr int kGroupDW = 4;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -226,7 +229,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
   CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW;
   bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, kBK, kBM) &&
-            make_map(&mW_k, BF, W, d, V, d * 2, kBK, kBN) &&
+            make_map(&mW_k, BF, W, d, V, d * 2, kBK, kBN / 2) &&
             make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
             make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, kBK, kBM) &&
             make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK) &&
@@ -254,9 +257,9 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.N = D.V;
   g.k_blocks = static_cast<int32_t>((d + kBK - 1) / kBK);
   g.k_row0 = 0;
-  g.m_blocks = static_cast<int32_t>((M + kBM - 1) / kBM);
+  g.m_blocks = static_cast<int32_t>((M + 2 * kBM - 1) / (2 * kBM));
   g.n_blocks = L.n_tiles_v;
-  g.group_m = kGroupM;
+  g.group_m = kGroupLogits;
   g.num_tiles = g.m_blocks * g.n_blocks;
   g.targets = targets;
   g.stats = ra.stats;
@@ -264,7 +267,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.V = D.V;
   g.flags = ra.flags;
   if (!mark(SOLO_STAGE_LOGITS) ||
-      fail(launch_gemm(kLogits, mX_k, mW_k, mP_st, g, std::min(g.num_tiles, sms), stream)))
+      fail(launch_gemm(kLogits, mX_k, mW_k, mP_st, g, sms, stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_LSE) || fail(launch_lse(ra, stream))) return SOLO_ERR_CUDA;
@@ -274,9 +277,10 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.N = D.d;
   gx.k_blocks = (D.V + kBK - 1) / kBK;
   gx.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
+  gx.group_m = kGroupDxhat;
   gx.num_tiles = gx.m_blocks * gx.n_blocks;
   if (!mark(SOLO_STAGE_DXHAT) ||
-      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, gx, std::min(gx.num_tiles, sms), stream)))
+      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, gx, sms, stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_norm_bwd(ra, stream, dgamma != nullptr)))
@@ -289,10 +293,11 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
     gw.N = D.d;
     gw.k_blocks = static_cast<int32_t>((D.N + kBK - 1) / kBK);
     gw.k_row0 = static_cast<int32_t>(static_cast<int64_t>(D.K - 1) * D.N);
-    gw.m_blocks = (D.V + kBM - 1) / kBM;
+    gw.m_blocks = (D.V + 2 * kBM - 1) / (2 * kBM);
     gw.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
+    gw.group_m = kGroupDW;
     gw.num_tiles = gw.m_blocks * gw.n_blocks;
-    if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, gw, std::min(gw.num_tiles, sms), stream)))
+    if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, gw, sms, stream)))
       return SOLO_ERR_CUDA;
   }
   if (!mark(SOLO_STAGE_DGAMMA)) return SOLO_ERR_CUDA;
