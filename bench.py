@@ -165,6 +165,29 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ----------------------------------------------------------------------- ranks
+
+def max_over_ranks(value: float, device=None) -> float:
+    """The largest value over all ranks (the slowest rank's time); identity at N=1."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank_step: int, steps: int, world: int, ms_max: float) -> float:
+    """Whole-job tokens/s: every rank's tokens over the slowest rank's time."""
+    return world * tokens_per_rank_step * steps / (ms_max / 1e3)
+
+
+def replica_workload(wl, rank: int):
+    """Rank r runs an independent replica of the workload with its own inputs."""
+    return wl.with_(seed=wl.seed + 1000 * rank) if rank else wl
+
+
 # ----------------------------------------------------------------------- CPU legs
 
 def oracle_sample(wl, rows: int, inp_rows=None):
@@ -273,7 +296,7 @@ def run_ours(args, wl):
     stream = torch.cuda.current_stream(dev)
 
     # inputs resident in HBM (seeded; ranks use distinct seeds: independent replicas)
-    wlr = wl.with_(seed=wl.seed + 1000 * rank) if rank else wl
+    wlr = replica_workload(wl, rank)
     inp = synth.generate(wlr)
     to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
         torch.bfloat16)
@@ -316,13 +339,9 @@ def run_ours(args, wl):
         stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(sr.SOLO_NUM_STAGES)]
     stage_ms /= args.steps
 
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-
+    ms = max_over_ranks(ms, dev)
     tokens_step = wl.M
-    value = world * tokens_step * args.steps / (ms / 1e3)
+    value = job_throughput(tokens_step, args.steps, world, ms)
 
     # ---- end to end through the C ABI with host buffers
     e2e = None
@@ -350,14 +369,10 @@ def run_ours(args, wl):
             e2e_step()
         t1.record(stream)
         barrier()
-        ems = t0.elapsed_time(t1)
-        if world > 1:
-            tt = torch.tensor([ems], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ems = float(tt.item())
+        ems = max_over_ranks(t0.elapsed_time(t1), dev)
         h2d = sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4
         d2h = lt_host.numel() * 4 + lm_host.numel() * 4
-        e2e = {"value": world * tokens_step * steps_e2e / (ems / 1e3), "unit": "tokens/s",
+        e2e = {"value": job_throughput(tokens_step, steps_e2e, world, ems), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     if rank != 0:

@@ -173,6 +173,19 @@ solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream
 /* Static description of a status code (never NULL). */
 const char* solo_readout_strerror(solo_status_t status);
 
+/*
+ * Self-test of the bounded waits that guard every pipeline wait in the
+ * library's kernels (a wait that does not complete gives up, sets
+ * SOLO_FLAG_TIMEOUT and lets the kernel return instead of hanging).  Launches
+ * one small kernel that waits on a barrier nothing arrives on, with a limit of
+ * limit_us microseconds (1 .. 1000000), through the same wait routine; the
+ * kernel then ORs SOLO_FLAG_TIMEOUT into *device_flags (a device uint32 the
+ * caller clears first) and returns.  Nothing faults or hangs; the context
+ * stays usable.  Asynchronous on `stream`.
+ */
+solo_status_t solo_readout_selftest_wait_timeout(uint32_t* device_flags, uint32_t limit_us,
+                                                 solo_stream_t stream);
+
 /* Library version, major * 10000 + minor * 100 + patch. */
 int32_t solo_readout_version(void);
 

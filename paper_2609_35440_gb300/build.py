@@ -1,6 +1,6 @@
 """Builds libsolo_readout.so in-tree with nvcc for sm_103a.
 
-The three translation units compile in parallel; the shared library links
+The translation units compile in parallel; the shared library links
 the CUDA runtime statically, so loading it needs no GPU and no libcuda
 (the driver is reached through the runtime's entry-point query at the
 first call).
@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIBDIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIBDIR, "libsolo_readout.so")
-SOURCES = ["gemm_tc.cu", "rowops.cu", "solo_readout.cu"]
+SOURCES = ["gemm_tc.cu", "rowops.cu", "solo_readout.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr"]

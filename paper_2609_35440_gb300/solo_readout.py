@@ -77,6 +77,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_fwd_bwd_static.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp, vp,
                                                  vp, ctypes.POINTER(vp), vp, vp, vp, vp]
     lib.solo_readout_fwd_bwd_static.restype = i32
+    lib.solo_readout_selftest_wait_timeout.argtypes = [vp, ctypes.c_uint32, vp]
+    lib.solo_readout_selftest_wait_timeout.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
     _lib = lib
@@ -184,6 +186,16 @@ def solo_readout_get_flags(workspace, stream=None) -> int:
     if st != SOLO_OK:
         raise SoloError(st, "solo_readout_get_flags")
     return out.value
+
+
+def solo_readout_selftest_wait_timeout(device_flags, limit_us: int, stream=None,
+                                       check: bool = True) -> int:
+    """Runs the bounded-wait self-test; SOLO_FLAG_TIMEOUT lands in device_flags."""
+    st = load().solo_readout_selftest_wait_timeout(_ptr(device_flags), int(limit_us),
+                                                   _stream_handle(stream))
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_selftest_wait_timeout")
+    return st
 
 
 def solo_readout_version() -> int:

@@ -125,3 +125,9 @@ def test_binding_has_no_fallback(tmp_path, monkeypatch):
     monkeypatch.setattr(solo_readout, "_lib", None)
     with pytest.raises(ImportError):
         solo_readout.load(str(tmp_path / "missing.so"))
+
+
+@pytest.mark.parametrize("flags,limit,want", [(None, 100, -1), (1 << 20, 0, -1),
+                                              (1 << 20, 2000000, -1), ((1 << 20) + 2, 100, -6)])
+def test_selftest_rejects_bad_arguments(sr, flags, limit, want):
+    assert sr.solo_readout_selftest_wait_timeout(flags, limit, stream=0, check=False) == want
