@@ -40,29 +40,73 @@ __device__ __forceinline__ bool token_kept(const RowArgs& a, int64_t row, int y)
 
 // ---- final RMSNorm: r_i = (mean_j h_ij^2 + eps)^-1/2, xhat = bf16(gamma h r) ------
 // The bf16 rounding of xhat is a quantisation decision, so it is taken on the
-// exact value: the sum of squares is accumulated error-free (each h^2 of a
-// bf16 h is exact in fp32; TwoSum keeps the rounding error of every add),
-// r is formed in fp64, and a product whose fp32 value lies within a few ulp
-// of a bf16 rounding midpoint is decided against the midpoint in fp64.
+// exact value, in fp32 arithmetic only (fp64 is slow on this part):
+//  - the sum of squares is accumulated error-free: each h^2 of a bf16 h is
+//    exact in fp32 and TwoSum keeps the rounding error of every addition
+//    (eight independent chains per lane, then pairwise across the warp), so
+//    the row's sum is an unevaluated pair (hi, lo) accurate to ~2^-46;
+//  - r = (ss/d + eps)^-1/2 comes from rsqrtf refined by one Newton step whose
+//    residual 1 - x r0^2 is formed with exact products (FMA), giving r as a
+//    pair (r32, r_lo) accurate to ~2^-44;
+//  - y = gamma h r is rounded from fp32 when it lies more than 4 ulp from a
+//    bf16 midpoint (|fl(gamma h r32) - y| <= 2 ulp); otherwise the sign of
+//    (y - midpoint) is decided from the exact product gamma h (r32 + r_lo).
 
-__device__ __forceinline__ uint16_t xhat_bf16(float gh, float r32, double r64) {
-  const float y = gh * r32;           // gh = gamma * h is exact in fp32
+struct F2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ F2 two_sum(float a, float b) {
+  const float s = a + b;
+  const float bb = s - a;
+  return {s, (a - (s - bb)) + (b - bb)};
+}
+
+// (a.hi + a.lo) + (b.hi + b.lo), renormalised
+__device__ __forceinline__ F2 add_f2(F2 a, F2 b) {
+  const F2 s = two_sum(a.hi, b.hi);
+  const float lo = s.lo + a.lo + b.lo;
+  const float hi = s.hi + lo;
+  return {hi, lo - (hi - s.hi)};
+}
+
+// (r32 + r_lo) ~= (x.hi + x.lo)^-1/2
+__device__ __forceinline__ F2 rsqrt_f2(F2 x) {
+  const float r0 = rsqrtf(x.hi);
+  const float q_hi = r0 * r0;
+  const float q_lo = fmaf(r0, r0, -q_hi);                // r0^2 = q_hi + q_lo exactly
+  const float p_hi = x.hi * q_hi;
+  const float p_lo = fmaf(x.hi, q_hi, -p_hi) + fmaf(x.hi, q_lo, x.lo * q_hi);
+  const float e = (1.0f - p_hi) - p_lo;                  // 1 - x r0^2 (tiny)
+  const float corr = 0.5f * r0 * e;                      // Newton: r = r0 (1 + e/2)
+  const float r32 = r0 + corr;
+  return {r32, corr - (r32 - r0)};
+}
+
+__device__ __forceinline__ uint16_t xhat_bf16(float gh, F2 r) {
+  const float y = gh * r.hi;          // gh = gamma * h is exact in fp32
   const uint32_t b = __float_as_uint(y);
   const uint32_t mag = b & 0x7FFFFFFFu;
   const int low = static_cast<int>(mag & 0xFFFFu) - 0x8000;
   if (low >= -4 && low <= 4 && mag < 0x7F000000u && mag >= 0x00800000u) {
-    // |y32 - y| <= 2 ulp, so the exact value lies strictly between the two
-    // neighbouring bf16 values; compare it with their midpoint.
+    // The exact value lies strictly between the two neighbouring bf16
+    // values; compare it with their midpoint.
     const uint32_t down = mag & 0xFFFF0000u;
-    const double mid = static_cast<double>(__uint_as_float(down | 0x8000u));
-    const double ya = fabs(static_cast<double>(gh) * r64);
+    const float mid = __uint_as_float(down | 0x8000u);
+    const float ga = fabsf(gh);
+    const float p_hi = ga * r.hi;
+    const float p_lo = fmaf(ga, r.hi, -p_hi) + ga * r.lo; // ga * (r.hi + r.lo) = p_hi + p_lo
+    const float dmid = (p_hi - mid) + p_lo;                // p_hi - mid is exact (close values)
     uint32_t q = down >> 16;
-    if (ya > mid || (ya == mid && (q & 1u))) q += 1;
+    if (dmid > 0.f || (dmid == 0.f && (q & 1u))) q += 1;
     return static_cast<uint16_t>(q | ((b >> 16) & 0x8000u));
   }
   return static_cast<uint16_t>((b + 0x7FFFu + ((b >> 16) & 1u)) >> 16);
 }
 
+// VPL > 0: the row is held in registers (VPL 16-byte vectors per lane, d <=
+// 256 * VPL), so h is read from memory once.  VPL == 0: any d, h re-read.
+template <int VPL>
 __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int lane = threadIdx.x & 31;
@@ -73,37 +117,73 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
   const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
   const int nv = a.d / 8;
-  float s = 0.f, c = 0.f;
-  for (int v = lane; v < nv; v += 32) {
+  constexpr int kCache = VPL > 0 ? VPL : 1;
+  uint4 hc[kCache];
+  // eight independent error-free sums (one per element position of a vector)
+  float s[8], c[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) s[j] = c[j] = 0.f;
+  auto accumulate = [&](const uint4& x) {
     float f[8];
-    unpack8(__ldg(h + v), f);
+    unpack8(x, f);
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float x = f[j] * f[j];
-      const float t = s + x;
-      const float bb = t - s;
-      c += (s - (t - bb)) + (x - bb);
-      s = t;
+      const float sq = f[j] * f[j];
+      const float t = s[j] + sq;
+      const float bb = t - s[j];
+      c[j] += (s[j] - (t - bb)) + (sq - bb);
+      s[j] = t;
     }
-  }
-  double ss = static_cast<double>(s) + static_cast<double>(c);
+  };
+  if constexpr (VPL > 0) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-  const double r64 = 1.0 / sqrt(ss / static_cast<double>(a.d) + static_cast<double>(a.eps));
-  const float r = static_cast<float>(r64);
+    for (int u = 0; u < VPL; ++u) {
+      const int v = lane + 32 * u;
+      hc[u] = v < nv ? __ldg(h + v) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < VPL; ++u) accumulate(hc[u]);
+  } else {
+    for (int v = lane; v < nv; v += 32) accumulate(__ldg(h + v));
+  }
+  F2 ss = {s[0], c[0]};
+#pragma unroll
+  for (int j = 1; j < 8; ++j) ss = add_f2(ss, F2{s[j], c[j]});
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const F2 other = {__shfl_xor_sync(0xffffffffu, ss.hi, o),
+                      __shfl_xor_sync(0xffffffffu, ss.lo, o)};
+    ss = add_f2(ss, other);
+  }
+  // x = ss / d + eps as a pair
+  const float fd = static_cast<float>(a.d);
+  const float m_hi = ss.hi / fd;
+  const float m_lo = (fmaf(-m_hi, fd, ss.hi) + ss.lo) / fd;
+  const F2 x = add_f2(F2{m_hi, m_lo}, F2{a.eps, 0.f});
+  const F2 rr = rsqrt_f2(x);
+  const float r = rr.hi;
   uint4* out = reinterpret_cast<uint4*>(a.xhat + row * a.d);
-  for (int v = lane; v < nv; v += 32) {
+  auto emit = [&](int v, const uint4& x) {
     float f[8], gg[8];
-    unpack8(__ldg(h + v), f);
+    unpack8(x, f);
     unpack8(__ldg(g + v), gg);
     uint32_t w[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const uint32_t lo = xhat_bf16(gg[2 * j] * f[2 * j], r, r64);
-      const uint32_t hi = xhat_bf16(gg[2 * j + 1] * f[2 * j + 1], r, r64);
+      const uint32_t lo = xhat_bf16(gg[2 * j] * f[2 * j], rr);
+      const uint32_t hi = xhat_bf16(gg[2 * j + 1] * f[2 * j + 1], rr);
       w[j] = lo | (hi << 16);
     }
     out[v] = make_uint4(w[0], w[1], w[2], w[3]);
+  };
+  if constexpr (VPL > 0) {
+#pragma unroll
+    for (int u = 0; u < VPL; ++u) {
+      const int v = lane + 32 * u;
+      if (v < nv) emit(v, hc[u]);
+    }
+  } else {
+    for (int v = lane; v < nv; v += 32) emit(v, __ldg(h + v));
   }
   if (lane == 0) a.r[row] = r;
 }
@@ -120,14 +200,19 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
   if (n < a.N) {
     const int64_t row = static_cast<int64_t>(k) * a.N + n;
     float mx = -INFINITY, s = 0.f;
-    for (int t = 0; t < a.n_tiles_v; ++t) {
-      const float2 st = a.stats[static_cast<int64_t>(t) * M + row];
-      if (st.x > mx) {
-        s = s * expf(mx - st.x) + st.y;
-        mx = st.x;
-      } else {
-        s += st.y * expf(st.x - mx);
-      }
+    for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
+      float2 st[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)         // independent loads, issued together
+        st[u] = t0 + u < a.n_tiles_v ? a.stats[static_cast<int64_t>(t0 + u) * M + row]
+                                     : make_float2(-INFINITY, 0.f);
+      float cm = mx;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) cm = fmaxf(cm, st[u].x);
+      s *= expf(mx - cm);                 // mx = -inf only before the first tile (s = 0)
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s += st[u].y * expf(st[u].x - cm);
+      mx = cm;
     }
     const float l = mx + logf(s);
     a.lse[row] = l;
@@ -235,6 +320,7 @@ __global__ void __launch_bounds__(256) grad_kernel(const RowArgs a) {
 
 // ---- RMSNorm backward: dh = r gamma dxhat - (r^3/d) h sum_l gamma_l dxhat_l h_l --
 
+template <int VPL>
 __global__ void __launch_bounds__(256) norm_bwd_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int lane = threadIdx.x & 31;
@@ -246,31 +332,59 @@ __global__ void __launch_bounds__(256) norm_bwd_kernel(const RowArgs a) {
   const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
   const float4* dx = reinterpret_cast<const float4*>(a.dxhat + row * a.d);
   const int nv = a.d / 8;
+  constexpr int kCache = VPL > 0 ? VPL : 1;
+  uint4 hc[kCache];
+  float4 d0c[kCache], d1c[kCache];
   float c = 0.f;
-  for (int v = lane; v < nv; v += 32) {
+  auto dot = [&](const uint4& hx, const uint4& gx, const float4& d0, const float4& d1) {
     float f[8], gg[8];
-    unpack8(__ldg(h + v), f);
-    unpack8(__ldg(g + v), gg);
-    const float4 d0 = dx[2 * v], d1 = dx[2 * v + 1];
+    unpack8(hx, f);
+    unpack8(gx, gg);
     c = fmaf(gg[0] * d0.x, f[0], c); c = fmaf(gg[1] * d0.y, f[1], c);
     c = fmaf(gg[2] * d0.z, f[2], c); c = fmaf(gg[3] * d0.w, f[3], c);
     c = fmaf(gg[4] * d1.x, f[4], c); c = fmaf(gg[5] * d1.y, f[5], c);
     c = fmaf(gg[6] * d1.z, f[6], c); c = fmaf(gg[7] * d1.w, f[7], c);
+  };
+  if constexpr (VPL > 0) {
+    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < VPL; ++u) {
+      const int v = lane + 32 * u;
+      const bool in = v < nv;
+      hc[u] = in ? __ldg(h + v) : make_uint4(0, 0, 0, 0);
+      d0c[u] = in ? dx[2 * v] : z4;
+      d1c[u] = in ? dx[2 * v + 1] : z4;
+    }
+#pragma unroll
+    for (int u = 0; u < VPL; ++u) {
+      const int v = lane + 32 * u;
+      if (v < nv) dot(hc[u], __ldg(g + v), d0c[u], d1c[u]);
+    }
+  } else {
+    for (int v = lane; v < nv; v += 32) dot(__ldg(h + v), __ldg(g + v), dx[2 * v], dx[2 * v + 1]);
   }
   c = warp_sum(c);
   const float r = a.r[row];
   const float coef = r * r * r * c / static_cast<float>(a.d);
   uint4* out = reinterpret_cast<uint4*>(a.dhidden[k] + n * a.d);
-  for (int v = lane; v < nv; v += 32) {
+  auto emit = [&](int v, const uint4& hx, const float4& d0, const float4& d1) {
     float f[8], gg[8];
-    unpack8(__ldg(h + v), f);
+    unpack8(hx, f);
     unpack8(__ldg(g + v), gg);
-    const float4 d0 = dx[2 * v], d1 = dx[2 * v + 1];
     const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
     float o[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) o[j] = fmaf(r * gg[j], dd[j], -coef * f[j]);
     out[v] = make_uint4(pack2(o[0], o[1]), pack2(o[2], o[3]), pack2(o[4], o[5]), pack2(o[6], o[7]));
+  };
+  if constexpr (VPL > 0) {
+#pragma unroll
+    for (int u = 0; u < VPL; ++u) {
+      const int v = lane + 32 * u;
+      if (v < nv) emit(v, hc[u], d0c[u], d1c[u]);
+    }
+  } else {
+    for (int v = lane; v < nv; v += 32) emit(v, __ldg(h + v), dx[2 * v], dx[2 * v + 1]);
   }
 }
 
@@ -303,9 +417,24 @@ __global__ void __launch_bounds__(256) dgamma_reduce_kernel(const RowArgs a) {
 
 }  // namespace
 
+// Smallest register cache (vectors per lane) that holds a row of d elements;
+// 0 (re-read the row) above d = 2048, where a larger cache costs more in
+// occupancy than the second read from L2 (measured at d = 2560).
+static int vectors_per_lane(int d) {
+  const int v = (d / 8 + 31) / 32;
+  return v <= 1 ? 1 : v <= 2 ? 2 : v <= 4 ? 4 : v <= 8 ? 8 : 0;
+}
+
 cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  rmsnorm_fwd_kernel<<<static_cast<unsigned>((M + 7) / 8), 256, 0, s>>>(a);
+  const unsigned grid = static_cast<unsigned>((M + 7) / 8);
+  switch (vectors_per_lane(a.d)) {
+    case 1: rmsnorm_fwd_kernel<1><<<grid, 256, 0, s>>>(a); break;
+    case 2: rmsnorm_fwd_kernel<2><<<grid, 256, 0, s>>>(a); break;
+    case 4: rmsnorm_fwd_kernel<4><<<grid, 256, 0, s>>>(a); break;
+    case 8: rmsnorm_fwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
+    default: rmsnorm_fwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
+  }
   return cudaGetLastError();
 }
 
@@ -331,7 +460,14 @@ cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
 
 cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  norm_bwd_kernel<<<static_cast<unsigned>((M + 7) / 8), 256, 0, s>>>(a);
+  const unsigned grid = static_cast<unsigned>((M + 7) / 8);
+  switch (vectors_per_lane(a.d)) {
+    case 1: norm_bwd_kernel<1><<<grid, 256, 0, s>>>(a); break;
+    case 2: norm_bwd_kernel<2><<<grid, 256, 0, s>>>(a); break;
+    case 4: norm_bwd_kernel<4><<<grid, 256, 0, s>>>(a); break;
+    case 8: norm_bwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
+    default: norm_bwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || !want_dgamma_parts) return e;
   dgamma_part_kernel<<<dim3((a.d + 255) / 256, a.dg_chunks), 256, 0, s>>>(a);
