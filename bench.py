@@ -40,6 +40,7 @@ sys.path.insert(0, ROOT)
 from paper_2609_35440_gb300 import costmodel, synth, workloads  # noqa: E402
 
 METRIC = "local-readout CE fwd+bwd tokens/s at d=2048,V=32000; % of bf16 tensor peak"
+EXIT_METRIC = "early-exit readout (forward: loss, top-1) tokens/s at d=2048,V=32000"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KERNEL_SOURCES = ["paper_2609_35440_gb300/csrc/gemm_tc.cu", "paper_2609_35440_gb300/csrc/ptx.cuh",
                   "paper_2609_35440_gb300/csrc/internal.h"]
@@ -57,6 +58,9 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--mode", default="train", choices=["train", "exit"],
+                   help="train: forward + backward (the headline); exit: forward-only "
+                        "early-exit readout (losses, top-1)")
     return p.parse_args()
 
 
@@ -424,6 +428,125 @@ def run_ours(args, wl):
         dist.destroy_process_group()
 
 
+def exit_oracle_sample(wl, rows: int, data):
+    import oracle.solo_oracle as orc
+    hidden, gamma, W, targets = data
+    orc.exit_readout([h[:rows] for h in hidden], gamma, W, targets[:, :rows],
+                     eps=float(np.float32(wl.eps)), ignore_index=wl.ignore_index)
+    return wl.K * rows
+
+
+def run_exit_bench(args, wl):
+    """The forward-only early-exit readout on the same workload (single GPU line)."""
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    from paper_2609_35440_gb300 import build
+    build.ensure_built()
+    sr.load()
+    dev = torch.device("cuda")
+    stream = torch.cuda.current_stream(dev)
+    inp = synth.generate(wl)
+    to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    hidden = [to_dev(inp.hidden[k]) for k in range(wl.K)]
+    gamma, W = to_dev(inp.gamma), to_dev(inp.W)
+    targets = torch.from_numpy(inp.targets).to(dev)
+    ex = sr.ExitReadout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index,
+                        device=dev)
+    clk = ClockSampler(dev.index).__enter__()
+    time.sleep(1.0)
+    for _ in range(max(args.warmup, 0)):
+        ex(hidden, gamma, W, targets, stream=stream)
+    torch.cuda.synchronize(dev)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(sr.SOLO_EXIT_NUM_STAGES + 1)]
+           for _ in range(args.steps)]
+    for evl in evs:
+        for e in evl:
+            e.record(stream)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for i in range(args.steps):
+        ex(hidden, gamma, W, targets, stream=stream, events=evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    clk.__exit__(None, None, None)
+    ms = t0.elapsed_time(t1)
+    stage_ms = np.zeros(sr.SOLO_EXIT_NUM_STAGES)
+    for evl in evs:
+        stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(sr.SOLO_EXIT_NUM_STAGES)]
+    stage_ms /= args.steps
+    flags = ex.flags(stream)
+    value = job_throughput(wl.M, args.steps, 1, ms)
+    # end to end: hidden states and targets from pinned host memory, losses and
+    # top-1 back to the host
+    h_host = [torch.from_numpy(np.ascontiguousarray(inp.hidden[k]).view(np.int16)).view(
+        torch.bfloat16).pin_memory() for k in range(wl.K)]
+    t_host = torch.from_numpy(inp.targets).pin_memory()
+    lt_host = torch.empty(wl.K, wl.N, dtype=torch.float32).pin_memory()
+    top_host = torch.empty(wl.K, wl.N, dtype=torch.int32).pin_memory()
+    steps_e2e = max(3, min(args.steps, 10))
+
+    def e2e_step():
+        for k in range(wl.K):
+            hidden[k].copy_(h_host[k], non_blocking=True)
+        targets.copy_(t_host, non_blocking=True)
+        ex(hidden, gamma, W, targets, stream=stream)
+        lt_host.copy_(ex.loss_tok, non_blocking=True)
+        top_host.copy_(ex.top1, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for _ in range(steps_e2e):
+        e2e_step()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ems = t0.elapsed_time(t1)
+    peaks, peak_src = load_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    G = costmodel.gemm_flops(wl.M, wl.V, wl.d)
+    achieved = G / (stage_ms[1] / 1e3) / 1e12
+    cpu = None
+    if not args.no_cpu:
+        data = prepare_oracle_sample(wl, 4096)
+        exit_oracle_sample(wl, 16, data)
+        t = time.perf_counter()
+        exit_oracle_sample(wl, 16, data)
+        per_row = (time.perf_counter() - t) / 16
+        rows = int(min(4096, max(16, args.cpu_seconds / max(per_row, 1e-9))))
+        t = time.perf_counter()
+        toks = exit_oracle_sample(wl, rows, data)
+        dt = time.perf_counter() - t
+        cpu = {"value": toks / dt, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+               "sample": f"first {rows} tokens of each of the {wl.K} modules, exit readout "
+                         f"(logits, log-sum-exp, argmax, losses) in fp64 numpy, {dt:.1f} s"}
+    line = {
+        "metric": EXIT_METRIC, "value": value, "unit": "tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "mode": "exit",
+        "config": {"workload": wl.name, "K": wl.K, "N": wl.N, "d": wl.d, "V": wl.V,
+                   "parallelism": "replicas1",
+                   "l2": "inputs larger than L2 (hidden+W 265 MB)"},
+        "stages_ms": {n: round(float(v), 4) for n, v in zip(sr.EXIT_STAGE_NAMES, stage_ms)},
+        "roofline": {"bound": "tensor", "kernel": "exit logits GEMM (tcgen05)",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "peak_source": f"{peak_src} bf16_tflops_sustained"},
+        "cpu_baseline": cpu,
+        "e2e": {"value": job_throughput(wl.M, steps_e2e, 1, ems), "unit": "tokens/s",
+                "h2d_bytes_per_step": sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4,
+                "d2h_bytes_per_step": lt_host.numel() * 4 + top_host.numel() * 4},
+        "clocks": clk.summary(),
+        "gpu_launches": 4 * args.steps,   # rmsnorm, exit GEMM, combine, module means
+        "device_flags": flags,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     wl = workload_from_name(args.workload)
@@ -431,6 +554,8 @@ def main():
         raise SystemExit("need --steps >= 1")
     if args.impl == "reference":
         run_reference(args, wl)
+    elif args.mode == "exit":
+        run_exit_bench(args, wl)
     else:
         run_ours(args, wl)
 

@@ -163,6 +163,69 @@ solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
                                           void* const* events, int32_t n_events);
 
 /*
+ * Early-exit readout, forward only: every module's hidden states decoded
+ * through the shared readout, as the exits of a trained SOLO model are (paper,
+ * Section 3 "Every module decodes" and Appendix E: each depth's next-token
+ * prediction, its log-probability and perplexity).  Per token: xhat =
+ * RMSNorm_gamma(h), z = W xhat, lse = logsumexp(z).
+ *
+ *  targets       int32 [K, N] or NULL (decoding only); same masking rules as
+ *                solo_readout_fwd_bwd.  Required when loss_tok or loss_mean is
+ *                given.
+ *  loss_tok      fp32 [K, N] or NULL: -log p(y) = lse - z_y, 0 when masked.
+ *  loss_mean     fp32 [K] or NULL: mean over kept tokens (exp gives the
+ *                module's perplexity).
+ *  top1          int32 [K, N] or NULL: argmax_v z, the first (lowest) index
+ *                among equal maxima.
+ *  top1_logprob  fp32 [K, N] or NULL: log p(top1) = max_v z - lse.
+ *  workspace     at least solo_readout_exit_workspace_bytes bytes.
+ *
+ * Runs the RMSNorm, one tensor-core pass over the vocabulary (K*2NVd FLOPs)
+ * and a combine; no exponential or gradient buffer is written.  Flags as for
+ * solo_readout_fwd_bwd (read with solo_readout_get_flags on this workspace).
+ */
+solo_status_t solo_readout_exit_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
+solo_status_t solo_readout_exit_forward(const solo_dims_t* dims,
+                                        const solo_bf16_t* const* hidden,
+                                        const solo_bf16_t* gamma,
+                                        const solo_bf16_t* W,
+                                        const int32_t* targets,
+                                        const uint8_t* mask,
+                                        float* loss_tok,
+                                        float* loss_mean,
+                                        int32_t* top1,
+                                        float* top1_logprob,
+                                        void* workspace, size_t workspace_bytes,
+                                        solo_stream_t stream);
+
+/* Stages of the exit readout, for solo_readout_exit_forward_events. */
+enum {
+  SOLO_EXIT_STAGE_RMSNORM = 0,  /* r_i and xhat                                      */
+  SOLO_EXIT_STAGE_LOGITS = 1,   /* tensor-core X W^T with per-tile max/sum/argmax     */
+  SOLO_EXIT_STAGE_COMBINE = 2,  /* logsumexp, top-1, losses, module means             */
+  SOLO_EXIT_NUM_STAGES = 3
+};
+
+/*
+ * Same as solo_readout_exit_forward, recording events[s] before stage s and
+ * events[SOLO_EXIT_NUM_STAGES] after the last (n_events must be
+ * SOLO_EXIT_NUM_STAGES + 1 caller-created cudaEvent_t handles).
+ */
+solo_status_t solo_readout_exit_forward_events(const solo_dims_t* dims,
+                                               const solo_bf16_t* const* hidden,
+                                               const solo_bf16_t* gamma,
+                                               const solo_bf16_t* W,
+                                               const int32_t* targets,
+                                               const uint8_t* mask,
+                                               float* loss_tok,
+                                               float* loss_mean,
+                                               int32_t* top1,
+                                               float* top1_logprob,
+                                               void* workspace, size_t workspace_bytes,
+                                               solo_stream_t stream,
+                                               void* const* events, int32_t n_events);
+
+/*
  * Waits for `stream`, then copies the flag word of the last call that used
  * `workspace` into *flags (host).  The word is cleared at the start of
  * every call.

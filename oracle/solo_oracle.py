@@ -181,6 +181,39 @@ def solo_readout_fwd_bwd(hidden, gamma, W, targets, mask=None, eps=1e-6,
     return out
 
 
+def exit_readout(hidden, gamma, W, targets=None, mask=None, eps=1e-6, ignore_index=-100,
+                 contract=True):
+    """Decoding through the shared readout at every depth (the early exits of
+    Section 3 and Appendix E): per token the first argmax of the logits and its
+    log-probability, and with targets the token loss -log p(y) (0 when masked)
+    and the mean over kept tokens of each module."""
+    K = len(hidden)
+    V = W.shape[0]
+    out = dict(top1=[], top1_logprob=[], loss_tok=[], loss_mean=np.zeros(K), z=[])
+    for k in range(K):
+        r, xhat = rmsnorm_forward(hidden[k], gamma, eps, contract)
+        z = logits(xhat, W)
+        lse = log_sum_exp(z)
+        top = np.argmax(z, axis=1)                 # first index among equal maxima
+        rows = np.arange(z.shape[0])
+        out["top1"].append(top)
+        out["top1_logprob"].append(z[rows, top] - lse)
+        out["z"].append(z)
+        if targets is not None:
+            kept, _ = kept_tokens(targets[k], None if mask is None else mask[k], V,
+                                  ignore_index)
+            y = np.asarray(targets[k])
+            loss = token_loss(z, lse, y, kept)
+            out["loss_tok"].append(loss)
+            n_valid = int(kept.sum())
+            out["loss_mean"][k] = loss.sum() / n_valid if n_valid else 0.0
+    out["top1"] = np.stack(out["top1"])
+    out["top1_logprob"] = np.stack(out["top1_logprob"])
+    if targets is not None:
+        out["loss_tok"] = np.stack(out["loss_tok"])
+    return out
+
+
 def final_module_chunked(h_rows_fn, N, gamma, W, y, kept, eps, contract=True,
                          dW_cols=None, chunk=1024):
     """Final-module pass over all N rows in chunks, for full-size checks.

@@ -26,6 +26,10 @@
 //           gradient, so the logits are never written and never recomputed.
 //  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3; fp32 out.
 //  kDW      dW = G^T Xhat over the final module's tokens; fp32 out.
+//  kExit    Z = Xhat W^T for the early exits (every depth decodes through the
+//           shared readout, paper Section 3 and Appendix E): per row and tile
+//           the max, the sum of exp(z - max) (online, one TMEM pass), the
+//           first column reaching the max and the target logit.
 //
 // Every wait is bounded (ptx.cuh); on a timeout all roles unwind, in-flight
 // copies and MMAs are drained, TMEM is freed and SOLO_FLAG_TIMEOUT is set.
@@ -87,7 +91,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmD, const GemmArgs args) {
   constexpr bool kAmn = (MODE == kDW);
-  constexpr bool kBmn = (MODE != kLogits);
+  constexpr bool kBmn = (MODE == kDxhat || MODE == kDW);
   constexpr uint32_t kIdesc = idesc_bf16_f32(kPairRows, kBN, kAmn, kBmn);
 
   extern __shared__ uint8_t smem_raw[];
@@ -274,7 +278,51 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const int row = m0 + 32 * q + lane;
       const int ncols = min(kBN, args.N - n0);    // valid columns, warp-uniform
 
-      if constexpr (MODE == kLogits) {
+      if constexpr (MODE == kExit) {
+        const bool row_ok = row < args.M;
+        const int y = (row_ok && args.targets) ? args.targets[row] : -1;
+        const int yrel = y - n0;
+        const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
+        float mx = -INFINITY, ssum = 0.f, zyv = 0.f;
+        int amax = 0;
+        for (int c = 0; c < kBN / 32; ++c) {
+          if (c * 32 >= ncols) break;
+          float v[32];
+          tmem_ld32(tbase + c * 32, v);
+          const int yc = has_y ? yrel - c * 32 : -1;
+          float cm = -INFINITY;
+          int ci = 0;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const bool in = c * 32 + j < ncols;
+            if (in && v[j] > cm) {          // strict: the first column reaching the max
+              cm = v[j];
+              ci = c * 32 + j;
+            }
+            zyv = (j == yc) ? v[j] : zyv;
+          }
+          if (cm > mx) {
+            ssum *= ex2_approx((mx - cm) * kLog2e);   // rescale to the new running max
+            mx = cm;
+            amax = ci;
+          }
+          const float mlog = mx * kLog2e;
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (c * 32 + j < ncols) ssum += ex2_approx(fmaf(v[j], kLog2e, -mlog));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (even) mbar_arrive(&tempty[acc]);
+          else mbar_arrive_remote(tempty_even + acc * 8);
+        }
+        if (row_ok) {
+          args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
+          args.argmax[static_cast<size_t>(nb) * args.M + row] = n0 + amax;
+        }
+        if (has_y) args.zy[row] = zyv;
+      } else if constexpr (MODE == kLogits) {
         const bool row_ok = row < args.M;
         const int y = row_ok ? args.targets[row] : -1;
         const int yrel = y - n0;
@@ -399,6 +447,7 @@ cudaError_t gemm_prepare(int /*device*/) {
   cudaError_t e = set_smem_attr<kLogits>();
   if (e == cudaSuccess) e = set_smem_attr<kDxhat>();
   if (e == cudaSuccess) e = set_smem_attr<kDW>();
+  if (e == cudaSuccess) e = set_smem_attr<kExit>();
   return e;
 }
 
@@ -417,6 +466,9 @@ cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& 
       break;
     case kDW:
       gemm_kernel<kDW><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      break;
+    case kExit:
+      gemm_kernel<kExit><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
       break;
   }
   return cudaGetLastError();

@@ -20,8 +20,10 @@ enum GemmMode : int {
   kLogits = 0,  // Z = Xhat W^T (A: Xhat K-major, B: W K-major); epilogue: per-tile
                 //   max / sum of exp, target logit, bf16 exp(z - tile max) stored
   kDxhat = 1,   // dXhat = G W (A: G K-major, B: W MN-major); epilogue: fp32 store
-  kDW = 2       // dW = G^T Xhat over the final module (A: G MN-major,
+  kDW = 2,      // dW = G^T Xhat over the final module (A: G MN-major,
                 //   B: Xhat MN-major); epilogue: fp32 store
+  kExit = 3     // Z = Xhat W^T for decoding only; epilogue: per-tile max, sum of
+                //   exp, first argmax, target logit; nothing else is stored
 };
 
 struct GemmArgs {
@@ -39,6 +41,7 @@ struct GemmArgs {
   float* zy;               // [M]: logit of the target
   int32_t V;
   uint32_t* flags;         // device flag word
+  int32_t* argmax;         // kExit: [n_blocks, M] first column of the tile maximum
 };
 
 size_t gemm_smem_bytes();
@@ -84,10 +87,16 @@ struct RowArgs {
   int32_t dg_rows;      // rows per dgamma chunk
   float* dgamma;        // [d] or null
   uint32_t* flags;
+  // exit readout
+  int32_t* argmax;       // [n_tiles_v, M]: first column of each tile's maximum
+  int32_t* top1;         // [M] or null: first argmax over the vocabulary
+  float* top1_logprob;   // [M] or null: log p of that entry
 };
 
 cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_lse(const RowArgs& a, cudaStream_t s);
+// The exit readout's combine: log-sum-exp, top-1, and (with targets) losses.
+cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts);
 cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s);

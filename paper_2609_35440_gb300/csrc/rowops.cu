@@ -190,6 +190,9 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
 
 // ---- log-sum-exp over column tiles, token loss, per-block module sums ----------
 
+// kExit: also the first argmax over the vocabulary and its log-probability;
+// targets may be absent (decoding only).
+template <bool kExit>
 __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
   const int k = blockIdx.y;
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
@@ -200,6 +203,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
   if (n < a.N) {
     const int64_t row = static_cast<int64_t>(k) * a.N + n;
     float mx = -INFINITY, s = 0.f;
+    int best_tile = 0;
     for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
       float2 st[8];
 #pragma unroll
@@ -208,15 +212,23 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
                                      : make_float2(-INFINITY, 0.f);
       float cm = mx;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) cm = fmaxf(cm, st[u].x);
+      for (int u = 0; u < 8; ++u) {
+        if (kExit && st[u].x > cm) best_tile = t0 + u;   // strict: the first tile with the max
+        cm = fmaxf(cm, st[u].x);
+      }
       s *= expf(mx - cm);                 // mx = -inf only before the first tile (s = 0)
 #pragma unroll
       for (int u = 0; u < 8; ++u) s += st[u].y * expf(st[u].x - cm);
       mx = cm;
     }
     const float l = mx + logf(s);
-    a.lse[row] = l;
-    const int y = a.targets[row];
+    if constexpr (kExit) {
+      if (a.top1) a.top1[row] = a.argmax[static_cast<int64_t>(best_tile) * M + row];
+      if (a.top1_logprob) a.top1_logprob[row] = mx - l;
+    } else {
+      a.lse[row] = l;
+    }
+    const int y = a.targets ? a.targets[row] : a.ignore_index;
     bad = !(y >= 0 && y < a.V) && y != a.ignore_index;
     const bool kept = token_kept(a, row, y);
     const float loss = kept ? l - a.zy[row] : 0.f;
@@ -271,7 +283,8 @@ __global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
   }
   if (threadIdx.x == 0) {
     const long long nv = sc[0];
-    a.loss_mean[k] = nv > 0 ? static_cast<float>(st[0] / static_cast<double>(nv)) : 0.f;
+    if (a.loss_mean)
+      a.loss_mean[k] = nv > 0 ? static_cast<float>(st[0] / static_cast<double>(nv)) : 0.f;
     a.inv_nvalid[k] = nv > 0 ? static_cast<float>(1.0 / static_cast<double>(nv)) : 0.f;
   }
 }
@@ -439,7 +452,15 @@ cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_lse(const RowArgs& a, cudaStream_t s) {
-  lse_kernel<<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+  lse_kernel<false><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  module_mean_kernel<<<a.K, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s) {
+  lse_kernel<true><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   module_mean_kernel<<<a.K, 256, 0, s>>>(a);

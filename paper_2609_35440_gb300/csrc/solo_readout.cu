@@ -306,6 +306,133 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   return SOLO_OK;
 }
 
+// ---- exit readout (forward only) --------------------------------------------------
+
+struct ExitLayout {
+  int64_t M = 0;
+  int n_tiles_v = 0;
+  int part_blocks = 0;
+  size_t flags = 0, r = 0, zy = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
+  size_t stats = 0, argmax = 0, xhat = 0, total = 0;
+};
+
+ExitLayout make_exit_layout(const solo_dims_t& d) {
+  ExitLayout L;
+  L.M = static_cast<int64_t>(d.K) * d.N;
+  L.n_tiles_v = (d.V + kBN - 1) / kBN;
+  L.part_blocks = static_cast<int>((d.N + 255) / 256);
+  const size_t M = static_cast<size_t>(L.M);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes, kAlign);
+    return at;
+  };
+  L.flags = take(256);
+  L.r = take(M * 4);
+  L.zy = take(M * 4);
+  L.part_sum = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
+  L.part_cnt = take(static_cast<size_t>(d.K) * L.part_blocks * 4);
+  L.inv_nvalid = take(SOLO_MAX_MODULES * 4);
+  L.stats = take(static_cast<size_t>(L.n_tiles_v) * M * 8);
+  L.argmax = take(static_cast<size_t>(L.n_tiles_v) * M * 4);
+  L.xhat = take(M * d.d * 2);
+  L.total = off;
+  return L;
+}
+
+solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                       const solo_bf16_t* gamma, const solo_bf16_t* W, const int32_t* targets,
+                       const uint8_t* mask, float* loss_tok, float* loss_mean, int32_t* top1,
+                       float* top1_logprob, void* workspace, size_t workspace_bytes,
+                       cudaStream_t stream, void* const* events, int32_t n_events) {
+  solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  const solo_dims_t& D = *dims;
+  if (hidden == nullptr || gamma == nullptr || W == nullptr || workspace == nullptr)
+    return SOLO_ERR_INVALID_ARG;
+  if (targets == nullptr && (loss_tok != nullptr || loss_mean != nullptr))
+    return SOLO_ERR_INVALID_ARG;     // losses need targets
+  if (events != nullptr && n_events != SOLO_EXIT_NUM_STAGES + 1) return SOLO_ERR_INVALID_ARG;
+  for (int k = 0; k < D.K; ++k) {
+    if (hidden[k] == nullptr) return SOLO_ERR_INVALID_ARG;
+    if (!aligned16(hidden[k])) return SOLO_ERR_MISALIGNED;
+  }
+  auto a4 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; };
+  if (!aligned16(gamma) || !aligned16(W) || !aligned16(workspace) || !a4(targets) ||
+      !a4(loss_tok) || !a4(loss_mean) || !a4(top1) || !a4(top1_logprob))
+    return SOLO_ERR_MISALIGNED;
+  const ExitLayout L = make_exit_layout(D);
+  if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+  int sms = 0;
+  st = device_setup(&sms);
+  if (st != SOLO_OK) return st;
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  RowArgs ra;
+  std::memset(&ra, 0, sizeof(ra));
+  for (int k = 0; k < D.K; ++k) ra.hidden[k] = hidden[k];
+  ra.N = D.N;
+  ra.K = D.K;
+  ra.d = D.d;
+  ra.V = D.V;
+  ra.n_tiles_v = L.n_tiles_v;
+  ra.ignore_index = D.ignore_index;
+  ra.eps = D.eps;
+  ra.gamma = gamma;
+  ra.targets = targets;
+  ra.mask = mask;
+  ra.r = reinterpret_cast<float*>(ws + L.r);
+  ra.xhat = reinterpret_cast<uint16_t*>(ws + L.xhat);
+  ra.zy = reinterpret_cast<float*>(ws + L.zy);
+  ra.stats = reinterpret_cast<float2*>(ws + L.stats);
+  ra.part_sum = reinterpret_cast<double*>(ws + L.part_sum);
+  ra.part_cnt = reinterpret_cast<int32_t*>(ws + L.part_cnt);
+  ra.part_blocks = L.part_blocks;
+  ra.inv_nvalid = reinterpret_cast<float*>(ws + L.inv_nvalid);
+  ra.loss_tok = loss_tok;
+  ra.loss_mean = loss_mean;
+  ra.flags = reinterpret_cast<uint32_t*>(ws + L.flags);
+  ra.argmax = reinterpret_cast<int32_t*>(ws + L.argmax);
+  ra.top1 = top1;
+  ra.top1_logprob = top1_logprob;
+
+  const uint64_t M = static_cast<uint64_t>(L.M);
+  const uint64_t d = static_cast<uint64_t>(D.d);
+  const uint64_t V = static_cast<uint64_t>(D.V);
+  CUtensorMap mX_k, mW_k;
+  if (!make_map(&mX_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ra.xhat, d, M, d * 2, kBK, kBM) ||
+      !make_map(&mW_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, W, d, V, d * 2, kBK, kBN / 2))
+    return SOLO_ERR_CUDA;
+  auto mark = [&](int stage) -> bool {
+    if (events == nullptr) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(events[stage]), stream) == cudaSuccess;
+  };
+  if (cudaMemsetAsync(ra.flags, 0, 256, stream) != cudaSuccess) return SOLO_ERR_CUDA;
+  if (!mark(0) || launch_rmsnorm_fwd(ra, stream) != cudaSuccess) return SOLO_ERR_CUDA;
+  GemmArgs g;
+  std::memset(&g, 0, sizeof(g));
+  g.M = static_cast<int32_t>(M);
+  g.N = D.V;
+  g.k_blocks = static_cast<int32_t>((d + kBK - 1) / kBK);
+  g.m_blocks = static_cast<int32_t>((M + 2 * kBM - 1) / (2 * kBM));
+  g.n_blocks = L.n_tiles_v;
+  g.group_m = kGroupLogits;
+  g.num_tiles = g.m_blocks * g.n_blocks;
+  g.targets = targets;
+  g.stats = ra.stats;
+  g.zy = ra.zy;
+  g.V = D.V;
+  g.flags = ra.flags;
+  g.argmax = ra.argmax;
+  // the store map is unused by this epilogue; any valid map fills the slot
+  if (!mark(1) || launch_gemm(kExit, mX_k, mW_k, mX_k, g, sms, stream) != cudaSuccess)
+    return SOLO_ERR_CUDA;
+  if (!mark(2) || launch_exit_lse(ra, stream) != cudaSuccess) return SOLO_ERR_CUDA;
+  if (!mark(3)) return SOLO_ERR_CUDA;
+  return SOLO_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -341,6 +468,37 @@ solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
   return run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
              workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), events,
              n_events);
+}
+
+solo_status_t solo_readout_exit_workspace_bytes(const solo_dims_t* dims, size_t* bytes) {
+  if (bytes == nullptr) return SOLO_ERR_INVALID_ARG;
+  const solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  *bytes = make_exit_layout(*dims).total;
+  return SOLO_OK;
+}
+
+solo_status_t solo_readout_exit_forward(const solo_dims_t* dims,
+                                        const solo_bf16_t* const* hidden,
+                                        const solo_bf16_t* gamma, const solo_bf16_t* W,
+                                        const int32_t* targets, const uint8_t* mask,
+                                        float* loss_tok, float* loss_mean, int32_t* top1,
+                                        float* top1_logprob, void* workspace,
+                                        size_t workspace_bytes, solo_stream_t stream) {
+  return run_exit(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, top1,
+                  top1_logprob, workspace, workspace_bytes,
+                  reinterpret_cast<cudaStream_t>(stream), nullptr, 0);
+}
+
+solo_status_t solo_readout_exit_forward_events(
+    const solo_dims_t* dims, const solo_bf16_t* const* hidden, const solo_bf16_t* gamma,
+    const solo_bf16_t* W, const int32_t* targets, const uint8_t* mask, float* loss_tok,
+    float* loss_mean, int32_t* top1, float* top1_logprob, void* workspace,
+    size_t workspace_bytes, solo_stream_t stream, void* const* events, int32_t n_events) {
+  if (events == nullptr) return SOLO_ERR_INVALID_ARG;
+  return run_exit(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, top1,
+                  top1_logprob, workspace, workspace_bytes,
+                  reinterpret_cast<cudaStream_t>(stream), events, n_events);
 }
 
 solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream,

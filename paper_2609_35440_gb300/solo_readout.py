@@ -28,6 +28,8 @@ SOLO_FLAG_BAD_TARGET = 1
 SOLO_FLAG_TIMEOUT = 2
 
 SOLO_NUM_STAGES = 8
+SOLO_EXIT_NUM_STAGES = 3
+EXIT_STAGE_NAMES = ["rmsnorm", "logits", "combine"]
 STAGE_NAMES = ["rmsnorm", "logits", "lse", "grad", "dxhat", "norm_bwd", "dW", "dgamma"]
 
 
@@ -79,6 +81,14 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_fwd_bwd_static.restype = i32
     lib.solo_readout_selftest_wait_timeout.argtypes = [vp, ctypes.c_uint32, vp]
     lib.solo_readout_selftest_wait_timeout.restype = i32
+    lib.solo_readout_exit_workspace_bytes.argtypes = [dims_p, ctypes.POINTER(sz)]
+    lib.solo_readout_exit_workspace_bytes.restype = i32
+    lib.solo_readout_exit_forward.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp, vp, vp,
+                                              vp, vp, vp, sz, vp]
+    lib.solo_readout_exit_forward.restype = i32
+    lib.solo_readout_exit_forward_events.argtypes = (
+        lib.solo_readout_exit_forward.argtypes + [ctypes.POINTER(vp), i32])
+    lib.solo_readout_exit_forward_events.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
     _lib = lib
@@ -178,6 +188,68 @@ def solo_readout_fwd_bwd_static(dims: solo_dims_t, hidden: Sequence, gamma, W, t
     if check and st != SOLO_OK:
         raise SoloError(st, "solo_readout_fwd_bwd_static")
     return st
+
+
+def solo_readout_exit_workspace_bytes(dims: solo_dims_t) -> int:
+    out = ctypes.c_size_t(0)
+    st = load().solo_readout_exit_workspace_bytes(ctypes.byref(dims), ctypes.byref(out))
+    if st != SOLO_OK:
+        raise SoloError(st, "solo_readout_exit_workspace_bytes")
+    return out.value
+
+
+def solo_readout_exit_forward(dims: solo_dims_t, hidden: Sequence, gamma, W, targets, mask,
+                              loss_tok, loss_mean, top1, top1_logprob, workspace,
+                              workspace_bytes: int | None = None, stream=None,
+                              check: bool = True, events=None) -> int:
+    """Early-exit readout (forward only): losses, top-1 and its log-probability per token.
+    With ``events`` (SOLO_EXIT_NUM_STAGES + 1 torch.cuda.Event) the _events entry point
+    is used and the stages are bracketed."""
+    K = dims.K
+    if len(hidden) != K:
+        raise ValueError("hidden needs K entries")
+    harr = (ctypes.c_void_p * K)(*[_ptr(h) for h in hidden])
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    args = [ctypes.byref(dims), harr, _ptr(gamma), _ptr(W), _ptr(targets), _ptr(mask),
+            _ptr(loss_tok), _ptr(loss_mean), _ptr(top1), _ptr(top1_logprob), _ptr(workspace),
+            int(workspace_bytes), _stream_handle(stream)]
+    if events is None:
+        st = load().solo_readout_exit_forward(*args)
+        name = "solo_readout_exit_forward"
+    else:
+        handles = [e.cuda_event if hasattr(e, "cuda_event") else int(e) for e in events]
+        arr = (ctypes.c_void_p * len(handles))(*handles)
+        st = load().solo_readout_exit_forward_events(*args, arr, len(handles))
+        name = "solo_readout_exit_forward_events"
+    if check and st != SOLO_OK:
+        raise SoloError(st, name)
+    return st
+
+
+class ExitReadout:
+    """Owns the outputs and workspace of the early-exit readout for one size."""
+
+    def __init__(self, K: int, N: int, d: int, V: int, eps: float = 1e-6,
+                 ignore_index: int = -100, with_targets: bool = True, device=None):
+        import torch
+        self.dims = make_dims(K, N, d, V, eps, ignore_index)
+        dev = torch.device("cuda" if device is None else device)
+        self.workspace = torch.empty(solo_readout_exit_workspace_bytes(self.dims),
+                                     dtype=torch.uint8, device=dev)
+        self.loss_tok = torch.empty(K, N, dtype=torch.float32, device=dev) if with_targets else None
+        self.loss_mean = torch.empty(K, dtype=torch.float32, device=dev) if with_targets else None
+        self.top1 = torch.empty(K, N, dtype=torch.int32, device=dev)
+        self.top1_logprob = torch.empty(K, N, dtype=torch.float32, device=dev)
+
+    def __call__(self, hidden, gamma, W, targets=None, mask=None, stream=None, events=None):
+        solo_readout_exit_forward(self.dims, hidden, gamma, W, targets, mask, self.loss_tok,
+                                  self.loss_mean, self.top1, self.top1_logprob,
+                                  self.workspace, stream=stream, events=events)
+        return self
+
+    def flags(self, stream=None) -> int:
+        return solo_readout_get_flags(self.workspace, stream)
 
 
 def solo_readout_get_flags(workspace, stream=None) -> int:

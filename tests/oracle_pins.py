@@ -284,3 +284,41 @@ def pin_init_statistics(orc):
 PINS = [pin_bf16_rounding, pin_zero_readout, pin_brute_force_ce, pin_finite_differences,
         pin_softmax_rows_sum_to_zero, pin_scale_invariance, pin_masking, pin_dgamma_identity,
         pin_torch_fp64, pin_row_subsets, pin_init_statistics]
+
+
+# -- early-exit readout ---------------------------------------------------------
+
+def pin_exit_readout(orc):
+    """Exits: brute-force argmax and log-probabilities; W = 0 decodes index 0 with
+    log p = -ln V; p(top1) >= p(y) with equality when the target is the argmax;
+    its losses equal the training call's."""
+    p = problem(K=2, N=6, d=8, V=20, seed=25, mask_frac=0.2, orc=orc)
+    p["W"] = p["W"] * 40.0
+    ex = orc.exit_readout(p["hidden"], p["gamma"], p["W"], p["targets"], eps=p["eps"],
+                          contract=False)
+    for k in range(p["K"]):
+        h = p["hidden"][k]
+        for i in range(p["N"]):
+            ms = sum(v * v for v in h[i]) / p["d"]
+            r = 1.0 / math.sqrt(ms + p["eps"])
+            x = [p["gamma"][j] * h[i][j] * r for j in range(p["d"])]
+            z = [sum(x[j] * p["W"][v][j] for j in range(p["d"])) for v in range(p["V"])]
+            best = max(range(p["V"]), key=lambda v: (z[v], -v))
+            assert ex["top1"][k][i] == best
+            lse = math.log(sum(math.exp(zv) for zv in z))
+            assert abs(ex["top1_logprob"][k][i] - (z[best] - lse)) < 1e-12
+            y = p["targets"][k][i]
+            if y >= 0:
+                assert ex["top1_logprob"][k][i] >= -ex["loss_tok"][k][i] - 1e-12
+                if y == best:
+                    assert abs(ex["top1_logprob"][k][i] + ex["loss_tok"][k][i]) < 1e-12
+    full = run(orc, p, contract=False)
+    np.testing.assert_allclose(ex["loss_tok"], full["loss_tok"], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(ex["loss_mean"], full["loss_mean"], rtol=0, atol=1e-13)
+    z0 = orc.exit_readout(p["hidden"], p["gamma"], np.zeros_like(p["W"]), None,
+                          eps=p["eps"], contract=True)
+    assert np.all(z0["top1"] == 0)
+    np.testing.assert_allclose(z0["top1_logprob"], -math.log(p["V"]), rtol=0, atol=1e-13)
+
+
+PINS.append(pin_exit_readout)

@@ -131,3 +131,20 @@ def test_binding_has_no_fallback(tmp_path, monkeypatch):
                                               (1 << 20, 2000000, -1), ((1 << 20) + 2, 100, -6)])
 def test_selftest_rejects_bad_arguments(sr, flags, limit, want):
     assert sr.solo_readout_selftest_wait_timeout(flags, limit, stream=0, check=False) == want
+
+
+def test_exit_readout_host_checks(sr):
+    fake = 1 << 20
+    dims = sr.make_dims(2, 16, 64, 100)
+    small = sr.solo_readout_exit_workspace_bytes(dims)
+    assert 0 < small < sr.solo_readout_workspace_bytes(dims)
+    # losses without targets, a missing hidden pointer, a small workspace
+    assert sr.solo_readout_exit_forward(dims, [fake, fake], fake, fake, None, None, fake, None,
+                                        fake, None, fake, workspace_bytes=1 << 30, stream=0,
+                                        check=False) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_exit_forward(dims, [fake, None], fake, fake, fake, None, None, None,
+                                        fake, None, fake, workspace_bytes=1 << 30, stream=0,
+                                        check=False) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_exit_forward(dims, [fake, fake], fake, fake, fake, None, None, None,
+                                        fake, None, fake, workspace_bytes=small - 1, stream=0,
+                                        check=False) == sr.SOLO_ERR_WORKSPACE_TOO_SMALL

@@ -149,6 +149,26 @@ def _mut_bad_target_not_masked(o):
     o.kept_tokens = f
 
 
+def _mut_exit_last_argmax(o):
+    orig = o.exit_readout
+
+    def f(*a, **kw):
+        out = orig(*a, **kw)
+        out["top1"] = np.stack([z.shape[1] - 1 - np.argmax(z[:, ::-1], axis=1) for z in out["z"]])
+        return out
+    o.exit_readout = f
+
+
+def _mut_exit_logprob_without_lse(o):
+    orig = o.exit_readout
+
+    def f(*a, **kw):
+        out = orig(*a, **kw)
+        out["top1_logprob"] = np.stack([np.max(z, axis=1) for z in out["z"]])
+        return out
+    o.exit_readout = f
+
+
 MUTATIONS = [v for k, v in sorted(globals().items()) if k.startswith("_mut_")]
 
 
