@@ -41,6 +41,8 @@ from paper_2609_35440_gb300 import costmodel, synth, workloads  # noqa: E402
 
 METRIC = "local-readout CE fwd+bwd tokens/s at d=2048,V=32000; % of bf16 tensor peak"
 EXIT_METRIC = "early-exit readout (forward: loss, top-1) tokens/s at d=2048,V=32000"
+HEADS_METRIC = ("local-readout CE fwd+bwd with head temperature and bias (+dtau, dbias) "
+                "tokens/s at d=2048,V=32000")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 KERNEL_SOURCES = ["paper_2609_35440_gb300/csrc/gemm_tc.cu", "paper_2609_35440_gb300/csrc/ptx.cuh",
                   "paper_2609_35440_gb300/csrc/internal.h"]
@@ -58,9 +60,10 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
-    p.add_argument("--mode", default="train", choices=["train", "exit"],
-                   help="train: forward + backward (the headline); exit: forward-only "
-                        "early-exit readout (losses, top-1)")
+    p.add_argument("--mode", default="train", choices=["train", "heads", "exit"],
+                   help="train: forward + backward (the headline); heads: the same with "
+                        "each head's temperature and bias and their gradients; exit: "
+                        "forward-only early-exit readout (losses, top-1)")
     return p.parse_args()
 
 
@@ -308,6 +311,11 @@ def run_ours(args, wl):
     gamma, W = to_dev(inp.gamma), to_dev(inp.W)
     targets = torch.from_numpy(inp.targets).to(dev)
     ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index, device=dev)
+    heads = {}
+    if args.mode == "heads":
+        tau, bias = synth.gen_heads(wlr)
+        heads = dict(tau=torch.from_numpy(tau).to(dev), bias=torch.from_numpy(bias).to(dev),
+                     head_grads=True)
     def barrier():
         if world > 1:
             dist.barrier()
@@ -316,7 +324,7 @@ def run_ours(args, wl):
     clk = ClockSampler(dev.index).__enter__()
     time.sleep(1.0)                      # let the sampler start before the warm-up
     for _ in range(max(args.warmup, 0)):
-        ro(hidden, gamma, W, targets, stream=stream)
+        ro(hidden, gamma, W, targets, stream=stream, **heads)
     barrier()
 
     # ---- device-resident timing of exactly `steps` calls; events recorded on the
@@ -332,7 +340,7 @@ def run_ours(args, wl):
     barrier()
     t0.record(stream)
     for i in range(args.steps):
-        ro(hidden, gamma, W, targets, stream=stream, events=step_evs[i])
+        ro(hidden, gamma, W, targets, stream=stream, events=step_evs[i], **heads)
     t1.record(stream)
     barrier()
     clk.__exit__(None, None, None)
@@ -361,7 +369,7 @@ def run_ours(args, wl):
             for k in range(wl.K):
                 hidden[k].copy_(h_host[k], non_blocking=True)
             targets.copy_(t_host, non_blocking=True)
-            ro(hidden, gamma, W, targets, stream=stream)
+            ro(hidden, gamma, W, targets, stream=stream, **heads)
             lt_host.copy_(ro.loss_tok, non_blocking=True)
             lm_host.copy_(ro.loss_mean, non_blocking=True)
 
@@ -399,12 +407,14 @@ def run_ours(args, wl):
     if not args.no_cpu:
         cpu = cpu_baseline(wl, args.cpu_seconds)
     # rmsnorm, logits, lse + module means, grad, dxhat, norm_bwd, dgamma parts, dW, dgamma
-    launches_per_step = 10
+    # (+ the bias-gradient reduction with heads)
+    launches_per_step = 11 if heads else 10
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "metric": HEADS_METRIC if heads else METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic",
+        "data": "synthetic", "mode": args.mode,
         "config": {"workload": wl.name, "K": wl.K, "N": wl.N, "d": wl.d, "V": wl.V,
                    "global_batch_tokens": world * wl.M, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (hidden+W 265 MB; 2.1 GB gradient buffer "

@@ -226,6 +226,47 @@ solo_status_t solo_readout_exit_forward_events(const solo_dims_t* dims,
                                                void* const* events, int32_t n_events);
 
 /*
+ * Each auxiliary head's own readout parameters (Algorithm 1): the local loss
+ * of module k is CE(softmax(tau_k W-bar xhat + b_k), y) and the terminal loss
+ * CE(softmax(W xhat + b), y).  All pointers are device pointers or NULL.
+ */
+typedef struct {
+  const float* tau;   /* [K] temperatures tau_k, or NULL for all 1; the terminal
+                         module's entry is normally 1 (the paper's terminal loss
+                         has none); its dW is the gradient for the given value */
+  const float* bias;  /* [K, V] biases: b_k for k < K-1 and the terminal b for
+                         k = K-1, or NULL for all 0 */
+  float* dtau;        /* [K] or NULL: dL_k/dtau_k = mean over kept tokens of
+                         E_p[s] - s_y, s = W-bar xhat (before tau and bias) */
+  float* dbias;       /* [K, V] or NULL: dL_k/db_k = sum over module k's tokens
+                         of (softmax - onehot) / Nvalid_k */
+} solo_heads_t;
+
+/*
+ * solo_readout_fwd_bwd with the heads' temperature and bias (Eq. 2 with tau_k;
+ * Algorithm 1's b_k and b).  heads == NULL is exactly solo_readout_fwd_bwd.
+ * dhidden, dW and dgamma include the factor tau_k of the chain rule.  events:
+ * NULL, or SOLO_NUM_STAGES + 1 cudaEvent_t handles recorded as in
+ * solo_readout_fwd_bwd_events (n_events must then be SOLO_NUM_STAGES + 1).
+ * The workspace size is the same as for solo_readout_fwd_bwd.
+ */
+solo_status_t solo_readout_fwd_bwd_heads(const solo_dims_t* dims,
+                                         const solo_bf16_t* const* hidden,
+                                         const solo_bf16_t* gamma,
+                                         const solo_bf16_t* W,
+                                         const int32_t* targets,
+                                         const uint8_t* mask,
+                                         const solo_heads_t* heads,
+                                         float* loss_tok,
+                                         float* loss_mean,
+                                         solo_bf16_t* const* dhidden,
+                                         float* dW,
+                                         float* dgamma,
+                                         void* workspace, size_t workspace_bytes,
+                                         solo_stream_t stream,
+                                         void* const* events, int32_t n_events);
+
+/*
  * Waits for `stream`, then copies the flag word of the last call that used
  * `workspace` into *flags (host).  The word is cleared at the start of
  * every call.

@@ -25,6 +25,12 @@ paragraph of Appendix D):
 8. final module only (Algorithm 1: only the terminal loss updates W):
    dW_vj = sum_i g_iv xhat_ij,   dgamma_j = sum_i dxhat_ij h_ij r_i
 
+With the heads' own parameters (Algorithm 1: the local loss of module k is
+CE(softmax(tau_k W-bar phi_k(h_k) + b_k), y), the terminal CE(W h_K + b, y))
+step 3 becomes z = tau_k s + b_k with s = xhat W^T, the chain rule puts tau_k
+in front of g in steps 6 and 8, and
+9. dtau_k = sum_i sum_v g_iv s_iv,   db_k = sum_i g_i   (per module).
+
 A token is kept when its target lies in [0, V), differs from ignore_index
 and its optional mask byte is non-zero.  A target outside [0, V) that is not
 ignore_index is treated as masked and reported (``bad_target``).
@@ -120,51 +126,66 @@ def rmsnorm_backward(dxhat, h, gamma, r):
             - (r ** 3 / d)[:, None] * h * c[:, None])
 
 
-def readout_grads(g, xhat, dxhat, h, r):
+def readout_grads(g, xhat, dxhat, h, r, tau=1.0):
     """(dW, dgamma) summed over the given rows of the final module."""
-    dW = g.T @ xhat
+    dW = tau * (g.T @ xhat)
     dgamma = np.sum(dxhat * h * r[:, None], axis=0)
     return dW, dgamma
 
 
 # -- drivers ----------------------------------------------------------------
 
-def module_rows(h, gamma, W, y, kept, n_valid, eps, contract=True):
+def head_logits(s, tau=1.0, b=None):
+    """z = tau s + b: a head's temperature and bias on the shared readout's logits."""
+    z = tau * s
+    return z if b is None else z + b[None, :]
+
+
+def module_rows(h, gamma, W, y, kept, n_valid, eps, contract=True, tau=1.0, b=None):
     """Every per-token quantity for a set of rows of one module."""
     r, xhat = rmsnorm_forward(h, gamma, eps, contract)
-    z = logits(xhat, W)
+    s = logits(xhat, W)
+    z = head_logits(s, tau, b)
     lse = log_sum_exp(z)
     loss = token_loss(z, lse, y, kept)
     g = logit_grad(z, lse, y, kept, n_valid)
-    dxhat = input_grad(g, W)
+    dxhat = tau * input_grad(g, W)
     dh = rmsnorm_backward(dxhat, h, gamma, r)
     zy = z[np.arange(len(y)), np.where(kept, y, 0)]
-    return dict(r=r, xhat=xhat, z=z, lse=lse, loss=loss, g=g, dxhat=dxhat,
-                dh=dh, zy=zy)
+    dtau = float(np.sum(g * s))
+    db = np.sum(g, axis=0)
+    return dict(r=r, xhat=xhat, s=s, z=z, lse=lse, loss=loss, g=g, dxhat=dxhat,
+                dh=dh, zy=zy, dtau=dtau, db=db, tau=tau)
 
 
 def solo_readout_fwd_bwd(hidden, gamma, W, targets, mask=None, eps=1e-6,
                          ignore_index=-100, contract=True, want_dW=True,
-                         want_dgamma=True):
+                         want_dgamma=True, tau=None, bias=None):
     """Full oracle for small problems.
 
     hidden: sequence of K float64 arrays [N, d]; gamma [d]; W [V, d];
     targets int [K, N]; mask None or [K, N].  Returns a dict with loss_tok
     [K, N], loss_mean [K], n_valid [K], dhidden (list of [N, d]), dW [V, d]
     and dgamma [d] of the final module, bad_target (bool) and per-module
-    intermediates ``rows`` (list of module_rows dicts).
+    intermediates ``rows`` (list of module_rows dicts).  With tau [K] and/or
+    bias [K, V] (the heads' parameters) also dtau [K] and dbias [K, V].
     """
     K = len(hidden)
     V = W.shape[0]
     out = dict(loss_tok=[], loss_mean=np.zeros(K), n_valid=np.zeros(K, int),
-               dhidden=[], rows=[], bad_target=False)
+               dhidden=[], rows=[], bad_target=False, dtau=np.zeros(K),
+               dbias=np.zeros((K, V)))
     for k in range(K):
         kept, bad = kept_tokens(targets[k], None if mask is None else mask[k],
                                 V, ignore_index)
         out["bad_target"] |= bool(bad.any())
         n_valid = int(kept.sum())
+        tk = 1.0 if tau is None else float(tau[k])
+        bk = None if bias is None else np.asarray(bias[k], dtype=np.float64)
         res = module_rows(hidden[k], gamma, W, np.asarray(targets[k]), kept,
-                          n_valid, eps, contract)
+                          n_valid, eps, contract, tau=tk, b=bk)
+        out["dtau"][k] = res["dtau"]
+        out["dbias"][k] = res["db"]
         out["loss_tok"].append(res["loss"])
         out["loss_mean"][k] = res["loss"].sum() / n_valid if n_valid else 0.0
         out["n_valid"][k] = n_valid
@@ -172,7 +193,7 @@ def solo_readout_fwd_bwd(hidden, gamma, W, targets, mask=None, eps=1e-6,
         out["rows"].append(res)
         if k == K - 1:
             dW, dgamma = readout_grads(res["g"], res["xhat"], res["dxhat"],
-                                       hidden[k], res["r"])
+                                       hidden[k], res["r"], tau=tk)
             if want_dW:
                 out["dW"] = dW
             if want_dgamma:

@@ -26,6 +26,9 @@
 //           gradient, so the logits are never written and never recomputed.
 //  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3; fp32 out.
 //  kDW      dW = G^T Xhat over the final module's tokens; fp32 out.
+//  kLogitsHeads  as kLogits with each head's temperature and bias (Algorithm
+//           1: z = tau_k W-bar xhat + b_k), plus per tile sum exp(z - m) s and
+//           the target's s, for the temperature's gradient.
 //  kExit    Z = Xhat W^T for the early exits (every depth decodes through the
 //           shared readout, paper Section 3 and Appendix E): per row and tile
 //           the max, the sum of exp(z - max) (online, one TMEM pass), the
@@ -322,12 +325,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           args.argmax[static_cast<size_t>(nb) * args.M + row] = n0 + amax;
         }
         if (has_y) args.zy[row] = zyv;
-      } else if constexpr (MODE == kLogits) {
+      } else if constexpr (MODE == kLogits || MODE == kLogitsHeads) {
+        constexpr bool kHeads = (MODE == kLogitsHeads);
         const bool row_ok = row < args.M;
         const int y = row_ok ? args.targets[row] : -1;
         const int yrel = y - n0;
         const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
-        float mx = -INFINITY, zyv = 0.f;
+        // z = tau s + b for this row's module (kHeads), z = s otherwise
+        float tau = 1.f;
+        const float* brow = nullptr;
+        if constexpr (kHeads) {
+          const int kmod = row_ok ? static_cast<int>(row / args.tokens_per_module) : 0;
+          if (args.tau) tau = args.tau[kmod];
+          if (args.bias) brow = args.bias + static_cast<size_t>(kmod) * args.V + n0;
+        }
+        auto affine = [&](float sv, int col) {
+          if constexpr (kHeads) return fmaf(tau, sv, (brow && col < ncols) ? brow[col] : 0.f);
+          return sv;
+        };
+        float mx = -INFINITY, zyv = 0.f, syv = 0.f;
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
           float v[32];
@@ -335,12 +351,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           const int yc = has_y ? yrel - c * 32 : -1;   // target column within this chunk
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            if (c * 32 + j < ncols) mx = fmaxf(mx, v[j]);
-            zyv = (j == yc) ? v[j] : zyv;
+            const float z = affine(v[j], c * 32 + j);
+            if (c * 32 + j < ncols) mx = fmaxf(mx, z);
+            zyv = (j == yc) ? z : zyv;
+            if constexpr (kHeads) syv = (j == yc) ? v[j] : syv;
           }
         }
         const float mlog = mx * kLog2e;
-        float ssum = 0.f;
+        float ssum = 0.f, usum = 0.f;
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
           if (lane == 0) bulk_wait_group_read<1>();
@@ -354,15 +372,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               tmem_ld32(tbase + c * 32, v);
             } else {
 #pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = -INFINITY;
+              for (int j = 0; j < 32; ++j) v[j] = 0.f;
             }
             uint32_t p[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               const int col = c * 32 + 2 * j;
-              const float e0 = col < ncols ? ex2_approx(fmaf(v[2 * j], kLog2e, -mlog)) : 0.f;
-              const float e1 = col + 1 < ncols ? ex2_approx(fmaf(v[2 * j + 1], kLog2e, -mlog)) : 0.f;
+              const float e0 =
+                  col < ncols ? ex2_approx(fmaf(affine(v[2 * j], col), kLog2e, -mlog)) : 0.f;
+              const float e1 =
+                  col + 1 < ncols ? ex2_approx(fmaf(affine(v[2 * j + 1], col + 1), kLog2e, -mlog))
+                                  : 0.f;
               ssum += e0 + e1;
+              if constexpr (kHeads) usum = fmaf(e0, v[2 * j], fmaf(e1, v[2 * j + 1], usum));
               p[j] = pack_bf16x2(e0, e1);
             }
 #pragma unroll
@@ -386,7 +408,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (even) mbar_arrive(&tempty[acc]);
           else mbar_arrive_remote(tempty_even + acc * 8);
         }
-        if (row_ok) args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
+        if (row_ok) {
+          args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
+          if constexpr (kHeads) args.usum[static_cast<size_t>(nb) * args.M + row] = usum;
+        }
+        if constexpr (kHeads) {
+          if (has_y) args.sy[row] = syv;
+        }
         if (has_y) args.zy[row] = zyv;
       } else {
         for (int c = 0; c < kBN / 32; ++c) {
@@ -448,6 +476,7 @@ cudaError_t gemm_prepare(int /*device*/) {
   if (e == cudaSuccess) e = set_smem_attr<kDxhat>();
   if (e == cudaSuccess) e = set_smem_attr<kDW>();
   if (e == cudaSuccess) e = set_smem_attr<kExit>();
+  if (e == cudaSuccess) e = set_smem_attr<kLogitsHeads>();
   return e;
 }
 
@@ -469,6 +498,9 @@ cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& 
       break;
     case kExit:
       gemm_kernel<kExit><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      break;
+    case kLogitsHeads:
+      gemm_kernel<kLogitsHeads><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
       break;
   }
   return cudaGetLastError();

@@ -22,8 +22,11 @@ enum GemmMode : int {
   kDxhat = 1,   // dXhat = G W (A: G K-major, B: W MN-major); epilogue: fp32 store
   kDW = 2,      // dW = G^T Xhat over the final module (A: G MN-major,
                 //   B: Xhat MN-major); epilogue: fp32 store
-  kExit = 3     // Z = Xhat W^T for decoding only; epilogue: per-tile max, sum of
+  kExit = 3,    // Z = Xhat W^T for decoding only; epilogue: per-tile max, sum of
                 //   exp, first argmax, target logit; nothing else is stored
+  kLogitsHeads = 4  // as kLogits with each head's temperature and bias applied,
+                    //   z = tau_k s + b_k (s = Xhat W^T), and per tile the sum of
+                    //   exp(z - m) s for the temperature's gradient
 };
 
 struct GemmArgs {
@@ -42,6 +45,12 @@ struct GemmArgs {
   int32_t V;
   uint32_t* flags;         // device flag word
   int32_t* argmax;         // kExit: [n_blocks, M] first column of the tile maximum
+  // kLogitsHeads
+  const float* tau;        // [K] or null (1)
+  const float* bias;       // [K, V] or null (0)
+  int64_t tokens_per_module;
+  float* usum;             // [n_blocks, M]: sum over the tile of exp(z - m) * s
+  float* sy;               // [M]: s at the target (before temperature and bias)
 };
 
 size_t gemm_smem_bytes();
@@ -91,12 +100,25 @@ struct RowArgs {
   int32_t* argmax;       // [n_tiles_v, M]: first column of each tile's maximum
   int32_t* top1;         // [M] or null: first argmax over the vocabulary
   float* top1_logprob;   // [M] or null: log p of that entry
+  // heads' temperature and bias
+  const float* tau;      // [K] or null
+  float* usum;           // [n_tiles_v, M] (with tau gradients)
+  float* sy;             // [M]
+  double* part_tau;      // [K, part_blocks]
+  float* dtau;           // [K] or null
+  float* dbias;          // [K, V] or null
+  float* db_part;        // [K, db_chunks, ldp]
+  int32_t db_chunks;     // row chunks per module of the gradient pass
 };
 
+constexpr int kGradRows = 256;   // rows per CTA of the gradient pass
+
 cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s);
-cudaError_t launch_lse(const RowArgs& a, cudaStream_t s);
+// heads: with the heads' temperature gradient (a.dtau) as well
+cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads = false);
 // The exit readout's combine: log-sum-exp, top-1, and (with targets) losses.
 cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s);
+// G in place; with a.dbias also the per-module column sums of dL/dz.
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts);
 cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s);

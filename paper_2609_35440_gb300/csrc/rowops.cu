@@ -190,35 +190,50 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
 
 // ---- log-sum-exp over column tiles, token loss, per-block module sums ----------
 
-// kExit: also the first argmax over the vocabulary and its log-probability;
-// targets may be absent (decoding only).
-template <bool kExit>
+enum LseKind { kLseTrain = 0, kLseExit = 1, kLseHeads = 2 };
+
+// kLseExit: also the first argmax over the vocabulary and its log-probability;
+// targets may be absent (decoding only).  kLseHeads: also the temperature's
+// gradient term E_p[s] - s_y of every kept token (s: logits before the
+// temperature and bias), summed per module like the loss.
+template <int kKind>
 __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
+  constexpr bool kExit = kKind == kLseExit;
+  constexpr bool kHeads = kKind == kLseHeads;
   const int k = blockIdx.y;
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int64_t n = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
-  double lsum = 0.0;
+  double lsum = 0.0, tsum = 0.0;
   int cnt = 0;
   int bad = 0;
   if (n < a.N) {
     const int64_t row = static_cast<int64_t>(k) * a.N + n;
-    float mx = -INFINITY, s = 0.f;
+    float mx = -INFINITY, s = 0.f, us = 0.f;
     int best_tile = 0;
     for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
       float2 st[8];
+      float uu[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)         // independent loads, issued together
-        st[u] = t0 + u < a.n_tiles_v ? a.stats[static_cast<int64_t>(t0 + u) * M + row]
-                                     : make_float2(-INFINITY, 0.f);
+      for (int u = 0; u < 8; ++u) {       // independent loads, issued together
+        const bool in = t0 + u < a.n_tiles_v;
+        st[u] = in ? a.stats[static_cast<int64_t>(t0 + u) * M + row] : make_float2(-INFINITY, 0.f);
+        if constexpr (kHeads) uu[u] = in ? a.usum[static_cast<int64_t>(t0 + u) * M + row] : 0.f;
+      }
       float cm = mx;
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         if (kExit && st[u].x > cm) best_tile = t0 + u;   // strict: the first tile with the max
         cm = fmaxf(cm, st[u].x);
       }
-      s *= expf(mx - cm);                 // mx = -inf only before the first tile (s = 0)
+      const float rescale = expf(mx - cm);  // mx = -inf only before the first tile (s = 0)
+      s *= rescale;
+      if constexpr (kHeads) us *= rescale;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) s += st[u].y * expf(st[u].x - cm);
+      for (int u = 0; u < 8; ++u) {
+        const float f = expf(st[u].x - cm);
+        s += st[u].y * f;
+        if constexpr (kHeads) us += uu[u] * f;
+      }
       mx = cm;
     }
     const float l = mx + logf(s);
@@ -235,49 +250,57 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     if (a.loss_tok) a.loss_tok[row] = loss;
     lsum = loss;
     cnt = kept ? 1 : 0;
+    if constexpr (kHeads) tsum = kept ? static_cast<double>(us / s - a.sy[row]) : 0.0;
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(a.flags, SOLO_FLAG_BAD_TARGET);
-  __shared__ double ssum[8];
+  __shared__ double ssum[8], stau[8];
   __shared__ int scnt[8];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    if constexpr (kHeads) tsum += __shfl_xor_sync(0xffffffffu, tsum, o);
   }
   if ((threadIdx.x & 31) == 0) {
     ssum[threadIdx.x >> 5] = lsum;
     scnt[threadIdx.x >> 5] = cnt;
+    stau[threadIdx.x >> 5] = tsum;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double t = 0.0;
+    double t = 0.0, tt = 0.0;
     int c = 0;
     for (int w = 0; w < 8; ++w) {
       t += ssum[w];
       c += scnt[w];
+      tt += stau[w];
     }
     a.part_sum[static_cast<int64_t>(k) * a.part_blocks + blockIdx.x] = t;
     a.part_cnt[static_cast<int64_t>(k) * a.part_blocks + blockIdx.x] = c;
+    if constexpr (kHeads) a.part_tau[static_cast<int64_t>(k) * a.part_blocks + blockIdx.x] = tt;
   }
 }
 
 __global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
   const int k = blockIdx.x;
-  double t = 0.0;
+  double t = 0.0, tt = 0.0;
   long long c = 0;
   for (int b = threadIdx.x; b < a.part_blocks; b += 256) {
     t += a.part_sum[static_cast<int64_t>(k) * a.part_blocks + b];
     c += a.part_cnt[static_cast<int64_t>(k) * a.part_blocks + b];
+    if (a.dtau) tt += a.part_tau[static_cast<int64_t>(k) * a.part_blocks + b];
   }
-  __shared__ double st[256];
+  __shared__ double st[256], stt[256];
   __shared__ long long sc[256];
   st[threadIdx.x] = t;
   sc[threadIdx.x] = c;
+  stt[threadIdx.x] = tt;
   __syncthreads();
   for (int o = 128; o > 0; o >>= 1) {
     if (threadIdx.x < o) {
       st[threadIdx.x] += st[threadIdx.x + o];
       sc[threadIdx.x] += sc[threadIdx.x + o];
+      stt[threadIdx.x] += stt[threadIdx.x + o];
     }
     __syncthreads();
   }
@@ -286,15 +309,18 @@ __global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
     if (a.loss_mean)
       a.loss_mean[k] = nv > 0 ? static_cast<float>(st[0] / static_cast<double>(nv)) : 0.f;
     a.inv_nvalid[k] = nv > 0 ? static_cast<float>(1.0 / static_cast<double>(nv)) : 0.f;
+    if (a.dtau) a.dtau[k] = nv > 0 ? static_cast<float>(stt[0] / static_cast<double>(nv)) : 0.f;
   }
 }
 
-// ---- dL/dz in place: G = (softmax - onehot) / Nvalid --------------------------
+// ---- dL/dz in place: G = tau (softmax - onehot) / Nvalid --------------------
 // The buffer holds p~ = bf16(exp(z - m_t)) for the column tile t of each
 // entry, so softmax = p~ * exp(m_t - lse).  The target entry is recomputed
 // from the fp32 target logit so that p_y - 1 keeps its relative precision.
 
-__global__ void __launch_bounds__(256) grad_kernel(const RowArgs a) {
+// One row per CTA: contiguous 16-byte vectors across the row (the fastest
+// form; used when no bias gradient is needed).
+__global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   extern __shared__ float ctile[];
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int64_t row = blockIdx.x;
@@ -306,7 +332,8 @@ __global__ void __launch_bounds__(256) grad_kernel(const RowArgs a) {
     for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
     return;
   }
-  const float w = a.inv_nvalid[k];
+  const float tau = a.tau ? a.tau[k] : 1.f;
+  const float w = a.inv_nvalid[k] * tau;
   const float l = a.lse[row];
   for (int t = threadIdx.x; t < a.n_tiles_v; t += 256)
     ctile[t] = expf(a.stats[static_cast<int64_t>(t) * M + row].x - l) * w;
@@ -329,6 +356,90 @@ __global__ void __launch_bounds__(256) grad_kernel(const RowArgs a) {
     }
     P[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
   }
+}
+
+// With the bias gradient: a CTA owns kGradRows rows of one module and 2048
+// columns (8 tiles), each thread one 8-column vector down those rows, so it
+// also sums dL/dz over its rows (fixed order, per row chunk).
+__global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
+  __shared__ float cfac[kGradRows][8];     // exp(m_t - lse) / Nvalid per row and tile
+  __shared__ float sgy[kGradRows];
+  __shared__ int sy[kGradRows];
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const int k = blockIdx.y / a.db_chunks;
+  const int chunk = blockIdx.y - k * a.db_chunks;
+  const int64_t row0 = static_cast<int64_t>(k) * a.N + static_cast<int64_t>(chunk) * kGradRows;
+  const int64_t left = static_cast<int64_t>(k + 1) * a.N - row0;
+  const int rows = left < kGradRows ? static_cast<int>(left) : kGradRows;
+  const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
+  const float w = a.inv_nvalid[k];
+  const float tau = a.tau ? a.tau[k] : 1.f;
+  if (threadIdx.x < rows) {
+    const int r = threadIdx.x;
+    const int64_t i = row0 + r;
+    const int y = a.targets[i];
+    const bool kept = token_kept(a, i, y);
+    const float l = a.lse[i];
+    const float wr = kept ? w : 0.f;
+#pragma unroll
+    for (int tt = 0; tt < 8; ++tt) {
+      const int t = t0 + tt;
+      cfac[r][tt] = (wr != 0.f && t < a.n_tiles_v)
+                        ? expf(a.stats[static_cast<int64_t>(t) * M + i].x - l) * wr : 0.f;
+    }
+    sgy[r] = kept ? (expf(a.zy[i] - l) - 1.0f) * wr : 0.f;
+    sy[r] = kept ? y : -1;
+  }
+  __syncthreads();
+  const int vec = blockIdx.x * 256 + threadIdx.x;    // 8-column vector of this thread
+  if (vec * 8 >= a.ldp) return;
+  const int col0 = vec * 8;
+  const int tt = threadIdx.x >> 5;                    // 32 vectors = one 256-column tile
+  float colsum[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) colsum[j] = 0.f;
+  uint4* P = reinterpret_cast<uint4*>(a.P + row0 * a.ldp) + vec;
+  const int64_t stride = a.ldp / 8;
+  constexpr int kAhead = 4;                           // rows in flight per thread
+  for (int r0 = 0; r0 < rows; r0 += kAhead) {
+    uint4 in[kAhead];
+#pragma unroll
+    for (int u = 0; u < kAhead; ++u)
+      if (r0 + u < rows) in[u] = P[(r0 + u) * stride];
+#pragma unroll
+    for (int u = 0; u < kAhead; ++u) {
+      const int r = r0 + u;
+      if (r >= rows) break;
+      const float c = cfac[r][tt];
+      const int ycol = sy[r] - col0;
+      float f[8];
+      unpack8(in[u], f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float g = f[j] * c;
+        if (j == ycol) g = sgy[r];
+        if (col0 + j >= a.V) g = 0.f;
+        colsum[j] += g;
+        f[j] = g * tau;
+      }
+      P[r * stride] =
+          make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+    }
+  }
+  float* out = a.db_part + (static_cast<int64_t>(k) * a.db_chunks + chunk) * a.ldp + col0;
+  reinterpret_cast<float4*>(out)[0] = make_float4(colsum[0], colsum[1], colsum[2], colsum[3]);
+  reinterpret_cast<float4*>(out)[1] = make_float4(colsum[4], colsum[5], colsum[6], colsum[7]);
+}
+
+// db_k[v] = sum over the row chunks of module k (fixed order)
+__global__ void __launch_bounds__(256) dbias_reduce_kernel(const RowArgs a) {
+  const int k = blockIdx.y;
+  const int v = blockIdx.x * 256 + threadIdx.x;
+  if (v >= a.V) return;
+  float acc = 0.f;
+  for (int c = 0; c < a.db_chunks; ++c)
+    acc += a.db_part[(static_cast<int64_t>(k) * a.db_chunks + c) * a.ldp + v];
+  a.dbias[static_cast<int64_t>(k) * a.V + v] = acc;
 }
 
 // ---- RMSNorm backward: dh = r gamma dxhat - (r^3/d) h sum_l gamma_l dxhat_l h_l --
@@ -451,8 +562,11 @@ cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse(const RowArgs& a, cudaStream_t s) {
-  lse_kernel<false><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads) {
+  if (heads)
+    lse_kernel<kLseHeads><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+  else
+    lse_kernel<kLseTrain><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   module_mean_kernel<<<a.K, 256, 0, s>>>(a);
@@ -460,7 +574,7 @@ cudaError_t launch_lse(const RowArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s) {
-  lse_kernel<true><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
+  lse_kernel<kLseExit><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   module_mean_kernel<<<a.K, 256, 0, s>>>(a);
@@ -468,14 +582,23 @@ cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
+  if (a.dbias) {
+    const dim3 grid((a.ldp / 8 + 255) / 256, a.K * a.db_chunks);
+    grad_colsum_kernel<<<grid, 256, 0, s>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dbias_reduce_kernel<<<dim3((a.V + 255) / 256, a.K), 256, 0, s>>>(a);
+    return cudaGetLastError();
+  }
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const size_t smem = static_cast<size_t>(a.n_tiles_v) * sizeof(float);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(grad_rows_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  grad_kernel<<<static_cast<unsigned>(M), 256, smem, s>>>(a);
+  grad_rows_kernel<<<static_cast<unsigned>(M), 256, smem, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -39,8 +39,10 @@ struct Layout {
   int n_tiles_v = 0;
   int part_blocks = 0;
   int dg_chunks = 0;
+  int db_chunks = 0;
   size_t flags = 0, r = 0, lse = 0, zy = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
-  size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0, total = 0;
+  size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0;
+  size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, total = 0;
 };
 
 solo_status_t check_dims(const solo_dims_t* d) {
@@ -63,6 +65,7 @@ Layout make_layout(const solo_dims_t& d) {
   L.n_tiles_v = (d.V + kBN - 1) / kBN;
   L.part_blocks = static_cast<int>((d.N + 255) / 256);
   L.dg_chunks = static_cast<int>((d.N + kDgRows - 1) / kDgRows);
+  L.db_chunks = static_cast<int>((d.N + kGradRows - 1) / kGradRows);
   const size_t M = static_cast<size_t>(L.M);
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -82,6 +85,11 @@ Layout make_layout(const solo_dims_t& d) {
   L.P = take(M * static_cast<size_t>(L.ldp) * 2);
   L.dxhat = take(M * d.d * 4);
   L.dgp = take(static_cast<size_t>(L.dg_chunks) * d.d * 4);
+  // heads' temperature and bias gradients
+  L.usum = take(static_cast<size_t>(L.n_tiles_v) * M * 4);
+  L.sy = take(M * 4);
+  L.part_tau = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
+  L.db_part = take(static_cast<size_t>(d.K) * L.db_chunks * L.ldp * 4);
   L.total = off;
   return L;
 }
@@ -155,10 +163,10 @@ bool make_map(CUtensorMap* m, CUtensorMapDataType dt, const void* ptr, uint64_t 
 
 solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
                   const solo_bf16_t* gamma, const solo_bf16_t* W, const int32_t* targets,
-                  const uint8_t* mask, float* loss_tok, float* loss_mean,
-                  solo_bf16_t* const* dhidden, float* dW, float* dgamma, void* workspace,
-                  size_t workspace_bytes, cudaStream_t stream, void* const* events,
-                  int32_t n_events) {
+                  const uint8_t* mask, const solo_heads_t* heads, float* loss_tok,
+                  float* loss_mean, solo_bf16_t* const* dhidden, float* dW, float* dgamma,
+                  void* workspace, size_t workspace_bytes, cudaStream_t stream,
+                  void* const* events, int32_t n_events) {
   // -------- host-side checks: nothing is enqueued when one fails
   solo_status_t st = check_dims(dims);
   if (st != SOLO_OK) return st;
@@ -177,6 +185,14 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
       (loss_tok && (reinterpret_cast<uintptr_t>(loss_tok) & 3u)) ||
       (reinterpret_cast<uintptr_t>(loss_mean) & 3u))
     return SOLO_ERR_MISALIGNED;
+  const float* tau = heads ? heads->tau : nullptr;
+  const float* bias = heads ? heads->bias : nullptr;
+  float* dtau = heads ? heads->dtau : nullptr;
+  float* dbias = heads ? heads->dbias : nullptr;
+  if ((reinterpret_cast<uintptr_t>(tau) & 3u) || (reinterpret_cast<uintptr_t>(bias) & 3u) ||
+      (reinterpret_cast<uintptr_t>(dtau) & 3u) || (reinterpret_cast<uintptr_t>(dbias) & 3u))
+    return SOLO_ERR_MISALIGNED;
+  const bool affine = tau || bias || dtau;   // z = tau s + b (and its temperature gradient)
   const Layout L = make_layout(D);
   if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
 
@@ -221,6 +237,14 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.dg_rows = kDgRows;
   ra.dgamma = dgamma;
   ra.flags = reinterpret_cast<uint32_t*>(ws + L.flags);
+  ra.tau = tau;
+  ra.usum = reinterpret_cast<float*>(ws + L.usum);
+  ra.sy = reinterpret_cast<float*>(ws + L.sy);
+  ra.part_tau = reinterpret_cast<double*>(ws + L.part_tau);
+  ra.dtau = dtau;
+  ra.dbias = dbias;
+  ra.db_part = reinterpret_cast<float*>(ws + L.db_part);
+  ra.db_chunks = L.db_chunks;
 
   const uint64_t M = static_cast<uint64_t>(L.M);
   const uint64_t d = static_cast<uint64_t>(D.d);
@@ -266,11 +290,17 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.zy = ra.zy;
   g.V = D.V;
   g.flags = ra.flags;
+  g.tau = tau;
+  g.bias = bias;
+  g.tokens_per_module = D.N;
+  g.usum = ra.usum;
+  g.sy = ra.sy;
   if (!mark(SOLO_STAGE_LOGITS) ||
-      fail(launch_gemm(kLogits, mX_k, mW_k, mP_st, g, sms, stream)))
+      fail(launch_gemm(affine ? kLogitsHeads : kLogits, mX_k, mW_k, mP_st, g, sms, stream)))
     return SOLO_ERR_CUDA;
 
-  if (!mark(SOLO_STAGE_LSE) || fail(launch_lse(ra, stream))) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_STAGE_LSE) || fail(launch_lse(ra, stream, dtau != nullptr)))
+    return SOLO_ERR_CUDA;
   if (!mark(SOLO_STAGE_GRAD) || fail(launch_grad(ra, stream))) return SOLO_ERR_CUDA;
 
   GemmArgs gx = g;
@@ -451,8 +481,23 @@ solo_status_t solo_readout_fwd_bwd(const solo_dims_t* dims, const solo_bf16_t* c
                                    float* loss_mean, solo_bf16_t* const* dhidden, float* dW,
                                    float* dgamma, void* workspace, size_t workspace_bytes,
                                    solo_stream_t stream) {
-  return run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
-             workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), nullptr, 0);
+  return run(dims, hidden, gamma, W, targets, mask, nullptr, loss_tok, loss_mean, dhidden, dW,
+             dgamma, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), nullptr,
+             0);
+}
+
+solo_status_t solo_readout_fwd_bwd_heads(const solo_dims_t* dims,
+                                         const solo_bf16_t* const* hidden,
+                                         const solo_bf16_t* gamma, const solo_bf16_t* W,
+                                         const int32_t* targets, const uint8_t* mask,
+                                         const solo_heads_t* heads, float* loss_tok,
+                                         float* loss_mean, solo_bf16_t* const* dhidden,
+                                         float* dW, float* dgamma, void* workspace,
+                                         size_t workspace_bytes, solo_stream_t stream,
+                                         void* const* events, int32_t n_events) {
+  return run(dims, hidden, gamma, W, targets, mask, heads, loss_tok, loss_mean, dhidden, dW,
+             dgamma, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), events,
+             events ? n_events : 0);
 }
 
 solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
@@ -465,8 +510,8 @@ solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
                                           solo_stream_t stream, void* const* events,
                                           int32_t n_events) {
   if (events == nullptr) return SOLO_ERR_INVALID_ARG;
-  return run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
-             workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), events,
+  return run(dims, hidden, gamma, W, targets, mask, nullptr, loss_tok, loss_mean, dhidden, dW,
+             dgamma, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), events,
              n_events);
 }
 
@@ -581,8 +626,8 @@ extern "C" solo_status_t solo_readout_fwd_bwd_static(
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // The launch sequence clears the flag word itself; every other scratch
   // buffer is written before it is read, so stale contents never leak.
-  st = run(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW, dgamma,
-           scratch, SOLO_STATIC_SCRATCH_BYTES, s, nullptr, 0);
+  st = run(dims, hidden, gamma, W, targets, mask, nullptr, loss_tok, loss_mean, dhidden, dW,
+           dgamma, scratch, SOLO_STATIC_SCRATCH_BYTES, s, nullptr, 0);
   if (st != SOLO_OK) return st;
   if (device_flags &&
       cudaMemcpyAsync(device_flags, scratch, sizeof(uint32_t), cudaMemcpyDeviceToDevice, s) !=

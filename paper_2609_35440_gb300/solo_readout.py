@@ -39,6 +39,11 @@ class solo_dims_t(ctypes.Structure):
                 ("ignore_index", ctypes.c_int32)]
 
 
+class solo_heads_t(ctypes.Structure):
+    _fields_ = [("tau", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("dtau", ctypes.c_void_p),
+                ("dbias", ctypes.c_void_p)]
+
+
 class SoloError(RuntimeError):
     def __init__(self, status: int, what: str):
         super().__init__(f"{what}: {strerror(status)} (status {status})")
@@ -89,6 +94,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_exit_forward_events.argtypes = (
         lib.solo_readout_exit_forward.argtypes + [ctypes.POINTER(vp), i32])
     lib.solo_readout_exit_forward_events.restype = i32
+    lib.solo_readout_fwd_bwd_heads.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp,
+                                                ctypes.POINTER(solo_heads_t), vp, vp,
+                                                ctypes.POINTER(vp), vp, vp, vp, sz, vp,
+                                                ctypes.POINTER(vp), i32]
+    lib.solo_readout_fwd_bwd_heads.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
     _lib = lib
@@ -252,6 +262,34 @@ class ExitReadout:
         return solo_readout_get_flags(self.workspace, stream)
 
 
+def solo_readout_fwd_bwd_heads(dims: solo_dims_t, hidden: Sequence, gamma, W, targets, mask,
+                               tau, bias, dtau, dbias, loss_tok, loss_mean,
+                               dhidden: Sequence, dW, dgamma, workspace,
+                               workspace_bytes: int | None = None, stream=None, events=None,
+                               check: bool = True) -> int:
+    """The call with each head's temperature tau [K] and bias [K, V] (either may be None)."""
+    K = dims.K
+    if len(hidden) != K or len(dhidden) != K:
+        raise ValueError("hidden and dhidden need K entries")
+    harr = (ctypes.c_void_p * K)(*[_ptr(h) for h in hidden])
+    darr = (ctypes.c_void_p * K)(*[_ptr(h) for h in dhidden])
+    heads = solo_heads_t(_ptr(tau), _ptr(bias), _ptr(dtau), _ptr(dbias))
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    if events is None:
+        earr, n = None, 0
+    else:
+        handles = [e.cuda_event if hasattr(e, "cuda_event") else int(e) for e in events]
+        earr, n = (ctypes.c_void_p * len(handles))(*handles), len(handles)
+    st = load().solo_readout_fwd_bwd_heads(
+        ctypes.byref(dims), harr, _ptr(gamma), _ptr(W), _ptr(targets), _ptr(mask),
+        ctypes.byref(heads), _ptr(loss_tok), _ptr(loss_mean), darr, _ptr(dW), _ptr(dgamma),
+        _ptr(workspace), int(workspace_bytes), _stream_handle(stream), earr, n)
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd_heads")
+    return st
+
+
 def solo_readout_get_flags(workspace, stream=None) -> int:
     out = ctypes.c_uint32(0)
     st = load().solo_readout_get_flags(_ptr(workspace), _stream_handle(stream), ctypes.byref(out))
@@ -290,9 +328,20 @@ class Readout:
         self.dhidden = [torch.empty(N, d, dtype=torch.bfloat16, device=dev) for _ in range(K)]
         self.dW = torch.empty(V, d, dtype=torch.float32, device=dev) if want_dW else None
         self.dgamma = torch.empty(d, dtype=torch.float32, device=dev) if want_dgamma else None
+        self.dtau = torch.empty(K, dtype=torch.float32, device=dev)
+        self.dbias = torch.empty(K, V, dtype=torch.float32, device=dev)
 
-    def __call__(self, hidden, gamma, W, targets, mask=None, stream=None, events=None):
-        if events is None:
+    def __call__(self, hidden, gamma, W, targets, mask=None, stream=None, events=None,
+                 tau=None, bias=None, head_grads=False):
+        """tau [K] / bias [K, V] (fp32, either may be None) select the heads' call;
+        head_grads also fills self.dtau and self.dbias."""
+        if tau is not None or bias is not None or head_grads:
+            solo_readout_fwd_bwd_heads(self.dims, hidden, gamma, W, targets, mask, tau, bias,
+                                       self.dtau if head_grads else None,
+                                       self.dbias if head_grads else None, self.loss_tok,
+                                       self.loss_mean, self.dhidden, self.dW, self.dgamma,
+                                       self.workspace, stream=stream, events=events)
+        elif events is None:
             solo_readout_fwd_bwd(self.dims, hidden, gamma, W, targets, mask, self.loss_tok,
                                  self.loss_mean, self.dhidden, self.dW, self.dgamma,
                                  self.workspace, stream=stream)

@@ -178,3 +178,17 @@ def random_mask(seed: int, K: int, N: int, frac: float) -> np.ndarray:
     for k in range(K):
         m[k, _perm_prefix(seed, S_MASK, N, int(round(frac * N)), 1000 + k)] = 0
     return m
+
+
+S_TAU, S_BIAS = 8, 9
+
+
+def gen_heads(wl: Workload, tau_spread: float = 0.5, bias_std: float = 0.5):
+    """Heads' parameters (fp32): temperatures tau_k = 1 + tau_spread * U(-1, 1) for
+    the auxiliary modules and 1 for the terminal; biases b_k ~ N(0, bias_std^2)."""
+    tau = (1.0 + tau_spread * (2.0 * uniform(wl.seed, S_TAU, 0, wl.K) - 1.0)).astype(np.float32)
+    tau[-1] = 1.0
+    bias = np.empty((wl.K, wl.V), dtype=np.float32)
+    for k in range(wl.K):
+        bias[k] = bias_std * normal(wl.seed, S_BIAS, 0, wl.V, sub=k)
+    return tau, bias

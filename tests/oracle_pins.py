@@ -322,3 +322,123 @@ def pin_exit_readout(orc):
 
 
 PINS.append(pin_exit_readout)
+
+
+# -- heads' temperature and bias ------------------------------------------------
+
+def _heads(p, seed=0):
+    rng = np.random.default_rng(seed)
+    tau = 0.5 + rng.random(p["K"])
+    bias = rng.normal(0.0, 0.7, size=(p["K"], p["V"]))
+    return tau, bias
+
+
+def pin_heads_finite_differences(orc):
+    """Central differences of every module loss in tau_k, b_k, h_k, and of the final
+    loss in W and gamma, with non-trivial temperatures and biases (exact mode)."""
+    p = problem(K=2, N=4, d=8, V=12, seed=27, mask_frac=0.25, row_scale=True, orc=orc)
+    p["W"] = p["W"] * 20.0
+    tau, bias = _heads(p, 1)
+    base = dict(tau=tau, bias=bias)
+    out = run(orc, p, contract=False, **base)
+    K, step = p["K"], 1e-6
+
+    def L(k, **over):
+        kw = dict(base)
+        kw.update({x: v for x, v in over.items() if x in ("tau", "bias")})
+        q = dict(p)
+        q.update({x: v for x, v in over.items() if x not in ("tau", "bias")})
+        return run(orc, q, contract=False, **kw)["loss_mean"][k]
+
+    for k in range(K):
+        tp, tm = tau.copy(), tau.copy()
+        tp[k] += step
+        tm[k] -= step
+        num = (L(k, tau=tp) - L(k, tau=tm)) / (2 * step)
+        assert abs(out["dtau"][k] - num) <= 1e-7 * max(1.0, abs(num)), ("dtau", k, out["dtau"][k], num)
+        numb = np.zeros(p["V"])
+        for v in range(p["V"]):
+            bp, bm = bias.copy(), bias.copy()
+            bp[k, v] += step
+            bm[k, v] -= step
+            numb[v] = (L(k, bias=bp) - L(k, bias=bm)) / (2 * step)
+        assert rel(out["dbias"][k], numb) < 1e-7, ("dbias", k, rel(out["dbias"][k], numb))
+        numh = np.zeros_like(p["hidden"][k])
+        for idx in np.ndindex(*numh.shape):
+            hp = [h.copy() for h in p["hidden"]]
+            hm = [h.copy() for h in p["hidden"]]
+            hp[k][idx] += step
+            hm[k][idx] -= step
+            numh[idx] = (L(k, hidden=hp) - L(k, hidden=hm)) / (2 * step)
+        assert rel(out["dhidden"][k], numh) < 1e-7, ("dH", k)
+    numW = np.zeros_like(p["W"])
+    for idx in np.ndindex(*numW.shape):
+        Wp, Wm = p["W"].copy(), p["W"].copy()
+        Wp[idx] += step
+        Wm[idx] -= step
+        numW[idx] = (L(K - 1, W=Wp) - L(K - 1, W=Wm)) / (2 * step)
+    assert rel(out["dW"], numW) < 1e-7, ("dW", rel(out["dW"], numW))
+
+
+def pin_heads_closed_forms(orc):
+    """W = 0: z = b, so loss = lse(b) - b_y, dtau = 0, db = mean over kept tokens of
+    softmax(b) - e_y; each db_k sums to zero; a constant added to b_k changes nothing."""
+    p = problem(K=2, N=9, d=8, V=16, seed=29, mask_frac=0.2, orc=orc)
+    tau, bias = _heads(p, 2)
+    p0 = dict(p, W=np.zeros_like(p["W"]))
+    out = run(orc, p0, contract=True, tau=tau, bias=bias)
+    for k in range(p["K"]):
+        kept, _ = orc.kept_tokens(p["targets"][k], None, p["V"], -100)
+        b = bias[k]
+        lse_b = math.log(sum(math.exp(x) for x in b))
+        prob = np.array([math.exp(x - lse_b) for x in b])
+        y = p["targets"][k]
+        for i in range(p["N"]):
+            want = lse_b - b[y[i]] if kept[i] else 0.0
+            assert abs(out["loss_tok"][k][i] - want) < 1e-12
+        assert abs(out["dtau"][k]) < 1e-15
+        want_db = np.zeros(p["V"])
+        for i in np.nonzero(kept)[0]:
+            want_db += prob
+            want_db[y[i]] -= 1.0
+        want_db /= kept.sum()
+        np.testing.assert_allclose(out["dbias"][k], want_db, rtol=0, atol=1e-13)
+    out = run(orc, p, contract=False, tau=tau, bias=bias)
+    assert np.max(np.abs(out["dbias"].sum(axis=1))) < 1e-14
+    shifted = run(orc, p, contract=False, tau=tau, bias=bias + np.array([[0.3], [-1.1]]))
+    np.testing.assert_allclose(shifted["loss_tok"], out["loss_tok"], rtol=0, atol=1e-12)
+    np.testing.assert_allclose(shifted["dtau"], out["dtau"], rtol=1e-10, atol=1e-14)
+    for k in range(p["K"]):
+        assert rel(shifted["dhidden"][k], out["dhidden"][k]) < 1e-10
+
+
+def pin_heads_torch_fp64(orc):
+    """tau and b as autograd leaves of F.rms_norm, matmul and F.cross_entropy."""
+    import torch
+    import torch.nn.functional as F
+    p = problem(K=3, N=7, d=16, V=30, seed=31, mask_frac=0.2, row_scale=True, orc=orc)
+    p["W"] = p["W"] * 5.0
+    tau, bias = _heads(p, 3)
+    out = run(orc, p, contract=False, tau=tau, bias=bias)
+    W = torch.tensor(p["W"], dtype=torch.float64, requires_grad=True)
+    g = torch.tensor(p["gamma"], dtype=torch.float64, requires_grad=True)
+    for k in range(p["K"]):
+        t = torch.tensor(tau[k], dtype=torch.float64, requires_grad=True)
+        b = torch.tensor(bias[k], dtype=torch.float64, requires_grad=True)
+        h = torch.tensor(p["hidden"][k], dtype=torch.float64, requires_grad=True)
+        y = torch.tensor(p["targets"][k], dtype=torch.int64)
+        x = F.rms_norm(h, (p["d"],), weight=g, eps=p["eps"])
+        loss = F.cross_entropy(t * (x @ W.T) + b, y, ignore_index=-100)
+        W.grad = None
+        g.grad = None
+        loss.backward()
+        assert abs(loss.item() - out["loss_mean"][k]) < 1e-12
+        assert abs(t.grad.item() - out["dtau"][k]) < 1e-12 * max(1.0, abs(t.grad.item()))
+        assert rel(out["dbias"][k], b.grad.numpy()) < 1e-11
+        assert rel(out["dhidden"][k], h.grad.numpy()) < 1e-11
+        if k == p["K"] - 1:
+            assert rel(out["dW"], W.grad.numpy()) < 1e-11
+            assert rel(out["dgamma"], g.grad.numpy()) < 1e-11
+
+
+PINS += [pin_heads_finite_differences, pin_heads_closed_forms, pin_heads_torch_fp64]

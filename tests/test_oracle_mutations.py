@@ -169,6 +169,41 @@ def _mut_exit_logprob_without_lse(o):
     o.exit_readout = f
 
 
+def _mut_heads_tau_missing_in_dh(o):
+    orig = o.module_rows
+
+    def f(h, gamma, W, y, kept, n_valid, eps, contract=True, tau=1.0, b=None):
+        res = orig(h, gamma, W, y, kept, n_valid, eps, contract, tau, b)
+        res["dxhat"] = o.input_grad(res["g"], W)
+        res["dh"] = o.rmsnorm_backward(res["dxhat"], h, gamma, res["r"])
+        return res
+    o.module_rows = f
+
+
+def _mut_heads_dtau_uses_z(o):
+    orig = o.module_rows
+
+    def f(h, gamma, W, y, kept, n_valid, eps, contract=True, tau=1.0, b=None):
+        res = orig(h, gamma, W, y, kept, n_valid, eps, contract, tau, b)
+        res["dtau"] = float(np.sum(res["g"] * res["z"]))
+        return res
+    o.module_rows = f
+
+
+def _mut_heads_db_times_tau(o):
+    orig = o.module_rows
+
+    def f(h, gamma, W, y, kept, n_valid, eps, contract=True, tau=1.0, b=None):
+        res = orig(h, gamma, W, y, kept, n_valid, eps, contract, tau, b)
+        res["db"] = tau * res["db"]
+        return res
+    o.module_rows = f
+
+
+def _mut_heads_bias_scaled_by_tau(o):
+    o.head_logits = lambda s, tau=1.0, b=None: tau * (s if b is None else s + b[None, :])
+
+
 MUTATIONS = [v for k, v in sorted(globals().items()) if k.startswith("_mut_")]
 
 
