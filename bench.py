@@ -41,6 +41,8 @@ from paper_2609_35440_gb300 import costmodel, synth, workloads  # noqa: E402
 
 METRIC = "local-readout CE fwd+bwd tokens/s at d=2048,V=32000; % of bf16 tensor peak"
 EXIT_METRIC = "early-exit readout (forward: loss, top-1) tokens/s at d=2048,V=32000"
+PRIVATE_METRIC = ("private readouts (PRIV) fwd+bwd with dW_k, dgamma_k for every module "
+                  "tokens/s at d=2048,V=32000")
 HEADS_METRIC = ("local-readout CE fwd+bwd with head temperature and bias (+dtau, dbias) "
                 "tokens/s at d=2048,V=32000")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
@@ -60,7 +62,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
-    p.add_argument("--mode", default="train", choices=["train", "heads", "exit"],
+    p.add_argument("--mode", default="train", choices=["train", "heads", "exit", "private"],
                    help="train: forward + backward (the headline); heads: the same with "
                         "each head's temperature and bias and their gradients; exit: "
                         "forward-only early-exit readout (losses, top-1)")
@@ -557,6 +559,64 @@ def run_exit_bench(args, wl):
     print(json.dumps(line), flush=True)
 
 
+def run_private_bench(args, wl):
+    """Private readouts: every module its own W_k and gain gamma_k (dW_k, dgamma_k)."""
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    from paper_2609_35440_gb300 import build
+    build.ensure_built()
+    sr.load()
+    dev = torch.device("cuda")
+    stream = torch.cuda.current_stream(dev)
+    inp = synth.generate(wl)
+    to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
+        torch.bfloat16)
+    K, N, d, V = wl.K, wl.N, wl.d, wl.V
+    hidden = [to_dev(inp.hidden[k]) for k in range(K)]
+    Ws = [to_dev(synth.gen_W(wl.with_(seed=wl.seed + 100 * k))) for k in range(K)]
+    gs = [to_dev(synth.gen_gamma(wl.with_(seed=wl.seed + 100 * k))) for k in range(K)]
+    targets = torch.from_numpy(inp.targets).to(dev)
+    dims = sr.make_dims(K, N, d, V, wl.eps, wl.ignore_index)
+    ws = torch.empty(sr.solo_readout_private_workspace_bytes(dims), dtype=torch.uint8, device=dev)
+    loss_tok = torch.empty(K, N, device=dev)
+    loss_mean = torch.empty(K, device=dev)
+    dh = [torch.empty(N, d, dtype=torch.bfloat16, device=dev) for _ in range(K)]
+    dW = [torch.empty(V, d, device=dev) for _ in range(K)]
+    dg = [torch.empty(d, device=dev) for _ in range(K)]
+    call = lambda: sr.solo_readout_fwd_bwd_private(dims, hidden, gs, Ws, targets, None, loss_tok,
+                                                   loss_mean, dh, dW, dg, ws, stream=stream)
+    clk = ClockSampler(dev.index).__enter__()
+    time.sleep(1.0)
+    for _ in range(max(args.warmup, 0)):
+        call()
+    torch.cuda.synchronize(dev)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        call()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    clk.__exit__(None, None, None)
+    ms = t0.elapsed_time(t1)
+    peaks, peak_src = load_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    algo = 3 * K * costmodel.gemm_flops(N, V, d)      # per module: logits, dX, dW_k
+    tflops = algo / (ms / args.steps / 1e3) / 1e12
+    line = {"metric": PRIVATE_METRIC, "value": job_throughput(wl.M, args.steps, 1, ms),
+            "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "mode": "private",
+            "config": {"workload": wl.name, "K": K, "N": N, "d": d, "V": V,
+                       "parallelism": "replicas1"},
+            "algo_tflops": tflops,
+            "algo_frac_of_peak": tflops / peak,
+            "peak_source": f"{peak_src} bf16_tflops_sustained",
+            "clocks": clk.summary(), "gpu_launches": 10 * K * args.steps,
+            "device_flags": sr.solo_readout_get_flags(ws, stream)}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     wl = workload_from_name(args.workload)
@@ -566,6 +626,8 @@ def main():
         run_reference(args, wl)
     elif args.mode == "exit":
         run_exit_bench(args, wl)
+    elif args.mode == "private":
+        run_private_bench(args, wl)
     else:
         run_ours(args, wl)
 

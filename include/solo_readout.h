@@ -267,6 +267,38 @@ solo_status_t solo_readout_fwd_bwd_heads(const solo_dims_t* dims,
                                          void* const* events, int32_t n_events);
 
 /*
+ * Private readouts (the paper's PRIV arm, Table "Readout sources") with a
+ * head-owned final norm: module k predicts through its own readout W_k and
+ * final RMSNorm gain gamma_k, both trained by its own loss, so every module
+ * gets dW_k and dgamma_k.  Each module is computed as a single-module
+ * problem; the modules run one after another on `stream`, sharing the
+ * workspace (solo_readout_private_workspace_bytes: the size for one module).
+ *
+ *  gamma, W   host arrays [K] of device pointers: gamma_k bf16 [d], W_k bf16 [V, d].
+ *  dW, dgamma host arrays [K] of device pointers (fp32 [V, d] / [d]); the
+ *             arrays or any entry may be NULL (not computed).
+ *  heads      as for solo_readout_fwd_bwd_heads (tau [K], bias [K, V], ...),
+ *             or NULL.
+ * Other arguments as for solo_readout_fwd_bwd.  Device flags of all modules
+ * accumulate in the workspace's flag word.
+ */
+solo_status_t solo_readout_private_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
+solo_status_t solo_readout_fwd_bwd_private(const solo_dims_t* dims,
+                                           const solo_bf16_t* const* hidden,
+                                           const solo_bf16_t* const* gamma,
+                                           const solo_bf16_t* const* W,
+                                           const int32_t* targets,
+                                           const uint8_t* mask,
+                                           const solo_heads_t* heads,
+                                           float* loss_tok,
+                                           float* loss_mean,
+                                           solo_bf16_t* const* dhidden,
+                                           float* const* dW,
+                                           float* const* dgamma,
+                                           void* workspace, size_t workspace_bytes,
+                                           solo_stream_t stream);
+
+/*
  * Waits for `stream`, then copies the flag word of the last call that used
  * `workspace` into *flags (host).  The word is cleared at the start of
  * every call.

@@ -235,6 +235,32 @@ def exit_readout(hidden, gamma, W, targets=None, mask=None, eps=1e-6, ignore_ind
     return out
 
 
+def solo_readout_private(hidden, gammas, Ws, targets, mask=None, eps=1e-6, ignore_index=-100,
+                         contract=True, tau=None, bias=None):
+    """Private readouts (the PRIV arm) with head-owned final norms: module k
+    predicts through its own W_k and gain gamma_k and gets dW_k, dgamma_k; each
+    module is the single-module problem of ``solo_readout_fwd_bwd``."""
+    K = len(hidden)
+    out = dict(loss_tok=[], loss_mean=np.zeros(K), dhidden=[], dW=[], dgamma=[],
+               dtau=np.zeros(K), dbias=[], bad_target=False)
+    for k in range(K):
+        r = solo_readout_fwd_bwd([hidden[k]], gammas[k], Ws[k], targets[k:k + 1],
+                                 None if mask is None else mask[k:k + 1], eps, ignore_index,
+                                 contract, tau=None if tau is None else tau[k:k + 1],
+                                 bias=None if bias is None else bias[k:k + 1])
+        out["loss_tok"].append(r["loss_tok"][0])
+        out["loss_mean"][k] = r["loss_mean"][0]
+        out["dhidden"].append(r["dhidden"][0])
+        out["dW"].append(r["dW"])
+        out["dgamma"].append(r["dgamma"])
+        out["dtau"][k] = r["dtau"][0]
+        out["dbias"].append(r["dbias"][0])
+        out["bad_target"] |= r["bad_target"]
+    out["loss_tok"] = np.stack(out["loss_tok"])
+    out["dbias"] = np.stack(out["dbias"])
+    return out
+
+
 def final_module_chunked(h_rows_fn, N, gamma, W, y, kept, eps, contract=True,
                          dW_cols=None, chunk=1024):
     """Final-module pass over all N rows in chunks, for full-size checks.

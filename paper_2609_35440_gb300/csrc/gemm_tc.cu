@@ -339,19 +339,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (args.tau) tau = args.tau[kmod];
           if (args.bias) brow = args.bias + static_cast<size_t>(kmod) * args.V + n0;
         }
-        auto affine = [&](float sv, int col) {
-          if constexpr (kHeads) return fmaf(tau, sv, (brow && col < ncols) ? brow[col] : 0.f);
-          return sv;
+        // bias of one 32-column chunk; rows of a tile share their module, so a
+        // warp's vector loads hit the same addresses
+        const bool bias_vec = (args.V & 3) == 0;
+        auto load_bias = [&](int c, float (&b)[32]) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) b[j] = 0.f;
+          if (!kHeads || brow == nullptr) return;
+          if (bias_vec && c * 32 + 32 <= ncols) {
+            const float4* b4 = reinterpret_cast<const float4*>(brow + c * 32);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+              const float4 t = __ldg(b4 + q4);
+              b[4 * q4] = t.x; b[4 * q4 + 1] = t.y; b[4 * q4 + 2] = t.z; b[4 * q4 + 3] = t.w;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (c * 32 + j < ncols) b[j] = __ldg(brow + c * 32 + j);
+          }
         };
         float mx = -INFINITY, zyv = 0.f, syv = 0.f;
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
-          float v[32];
+          float v[32], bb[32];
           tmem_ld32(tbase + c * 32, v);
+          if constexpr (kHeads) load_bias(c, bb);
           const int yc = has_y ? yrel - c * 32 : -1;   // target column within this chunk
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            const float z = affine(v[j], c * 32 + j);
+            const float z = kHeads ? fmaf(tau, v[j], bb[j]) : v[j];
             if (c * 32 + j < ncols) mx = fmaxf(mx, z);
             zyv = (j == yc) ? z : zyv;
             if constexpr (kHeads) syv = (j == yc) ? v[j] : syv;
@@ -367,22 +384,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
           for (int half = 0; half < 2; ++half) {
             const int c = 2 * cp + half;
-            float v[32];
+            float v[32], bb[32];
             if (c * 32 < ncols) {
               tmem_ld32(tbase + c * 32, v);
+              if constexpr (kHeads) load_bias(c, bb);
             } else {
 #pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = 0.f;
+              for (int j = 0; j < 32; ++j) v[j] = bb[j] = 0.f;
             }
             uint32_t p[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               const int col = c * 32 + 2 * j;
-              const float e0 =
-                  col < ncols ? ex2_approx(fmaf(affine(v[2 * j], col), kLog2e, -mlog)) : 0.f;
-              const float e1 =
-                  col + 1 < ncols ? ex2_approx(fmaf(affine(v[2 * j + 1], col + 1), kLog2e, -mlog))
-                                  : 0.f;
+              const float z0 = kHeads ? fmaf(tau, v[2 * j], bb[2 * j]) : v[2 * j];
+              const float z1 = kHeads ? fmaf(tau, v[2 * j + 1], bb[2 * j + 1]) : v[2 * j + 1];
+              const float e0 = col < ncols ? ex2_approx(fmaf(z0, kLog2e, -mlog)) : 0.f;
+              const float e1 = col + 1 < ncols ? ex2_approx(fmaf(z1, kLog2e, -mlog)) : 0.f;
               ssum += e0 + e1;
               if constexpr (kHeads) usum = fmaf(e0, v[2 * j], fmaf(e1, v[2 * j + 1], usum));
               p[j] = pack_bf16x2(e0, e1);

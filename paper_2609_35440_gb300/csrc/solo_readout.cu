@@ -166,7 +166,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
                   const uint8_t* mask, const solo_heads_t* heads, float* loss_tok,
                   float* loss_mean, solo_bf16_t* const* dhidden, float* dW, float* dgamma,
                   void* workspace, size_t workspace_bytes, cudaStream_t stream,
-                  void* const* events, int32_t n_events) {
+                  void* const* events, int32_t n_events, bool clear_flags = true) {
   // -------- host-side checks: nothing is enqueued when one fails
   solo_status_t st = check_dims(dims);
   if (st != SOLO_OK) return st;
@@ -271,7 +271,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   };
   auto fail = [](cudaError_t e) { return e != cudaSuccess; };
 
-  if (fail(cudaMemsetAsync(ra.flags, 0, 256, stream))) return SOLO_ERR_CUDA;
+  if (clear_flags && fail(cudaMemsetAsync(ra.flags, 0, 256, stream))) return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_RMSNORM) || fail(launch_rmsnorm_fwd(ra, stream))) return SOLO_ERR_CUDA;
 
@@ -544,6 +544,57 @@ solo_status_t solo_readout_exit_forward_events(
   return run_exit(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, top1,
                   top1_logprob, workspace, workspace_bytes,
                   reinterpret_cast<cudaStream_t>(stream), events, n_events);
+}
+
+solo_status_t solo_readout_private_workspace_bytes(const solo_dims_t* dims, size_t* bytes) {
+  if (bytes == nullptr) return SOLO_ERR_INVALID_ARG;
+  solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  solo_dims_t one = *dims;
+  one.K = 1;
+  *bytes = make_layout(one).total;
+  return SOLO_OK;
+}
+
+solo_status_t solo_readout_fwd_bwd_private(
+    const solo_dims_t* dims, const solo_bf16_t* const* hidden, const solo_bf16_t* const* gamma,
+    const solo_bf16_t* const* W, const int32_t* targets, const uint8_t* mask,
+    const solo_heads_t* heads, float* loss_tok, float* loss_mean, solo_bf16_t* const* dhidden,
+    float* const* dW, float* const* dgamma, void* workspace, size_t workspace_bytes,
+    solo_stream_t stream) {
+  solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  const solo_dims_t D = *dims;
+  if (hidden == nullptr || gamma == nullptr || W == nullptr || dhidden == nullptr ||
+      targets == nullptr || loss_mean == nullptr)
+    return SOLO_ERR_INVALID_ARG;
+  for (int k = 0; k < D.K; ++k)
+    if (gamma[k] == nullptr || W[k] == nullptr || hidden[k] == nullptr || dhidden[k] == nullptr)
+      return SOLO_ERR_INVALID_ARG;
+  solo_dims_t one = D;
+  one.K = 1;
+  if (workspace_bytes < make_layout(one).total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+  // Every module is its own single-module problem: its head's readout W_k and
+  // final-norm gain gamma_k, with dW_k and dgamma_k.  The modules run one after
+  // another on `stream` and share the workspace; device flags accumulate.
+  const int64_t N = D.N;
+  for (int k = 0; k < D.K; ++k) {
+    solo_heads_t hk{};
+    const solo_heads_t* hp = nullptr;
+    if (heads) {
+      hk.tau = heads->tau ? heads->tau + k : nullptr;
+      hk.bias = heads->bias ? heads->bias + static_cast<int64_t>(k) * D.V : nullptr;
+      hk.dtau = heads->dtau ? heads->dtau + k : nullptr;
+      hk.dbias = heads->dbias ? heads->dbias + static_cast<int64_t>(k) * D.V : nullptr;
+      hp = &hk;
+    }
+    st = run(&one, hidden + k, gamma[k], W[k], targets + k * N, mask ? mask + k * N : nullptr,
+             hp, loss_tok ? loss_tok + k * N : nullptr, loss_mean + k, dhidden + k,
+             dW ? dW[k] : nullptr, dgamma ? dgamma[k] : nullptr, workspace, workspace_bytes,
+             reinterpret_cast<cudaStream_t>(stream), nullptr, 0, /*clear_flags=*/k == 0);
+    if (st != SOLO_OK) return st;
+  }
+  return SOLO_OK;
 }
 
 solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream,

@@ -99,6 +99,14 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                                 ctypes.POINTER(vp), vp, vp, vp, sz, vp,
                                                 ctypes.POINTER(vp), i32]
     lib.solo_readout_fwd_bwd_heads.restype = i32
+    lib.solo_readout_private_workspace_bytes.argtypes = [dims_p, ctypes.POINTER(sz)]
+    lib.solo_readout_private_workspace_bytes.restype = i32
+    lib.solo_readout_fwd_bwd_private.argtypes = [dims_p, ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                                  ctypes.POINTER(vp), vp, vp,
+                                                  ctypes.POINTER(solo_heads_t), vp, vp,
+                                                  ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                                  ctypes.POINTER(vp), vp, sz, vp]
+    lib.solo_readout_fwd_bwd_private.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
     _lib = lib
@@ -287,6 +295,36 @@ def solo_readout_fwd_bwd_heads(dims: solo_dims_t, hidden: Sequence, gamma, W, ta
         _ptr(workspace), int(workspace_bytes), _stream_handle(stream), earr, n)
     if check and st != SOLO_OK:
         raise SoloError(st, "solo_readout_fwd_bwd_heads")
+    return st
+
+
+def solo_readout_private_workspace_bytes(dims: solo_dims_t) -> int:
+    out = ctypes.c_size_t(0)
+    st = load().solo_readout_private_workspace_bytes(ctypes.byref(dims), ctypes.byref(out))
+    if st != SOLO_OK:
+        raise SoloError(st, "solo_readout_private_workspace_bytes")
+    return out.value
+
+
+def solo_readout_fwd_bwd_private(dims: solo_dims_t, hidden: Sequence, gammas: Sequence,
+                                 Ws: Sequence, targets, mask, loss_tok, loss_mean,
+                                 dhidden: Sequence, dWs, dgammas, workspace, tau=None, bias=None,
+                                 dtau=None, dbias=None, workspace_bytes: int | None = None,
+                                 stream=None, check: bool = True) -> int:
+    """Private readouts W_k and head-owned gains gamma_k: dW_k and dgamma_k for every module."""
+    K = dims.K
+    arr = lambda xs: None if xs is None else (ctypes.c_void_p * K)(*[_ptr(x) for x in xs])
+    heads = None
+    if any(x is not None for x in (tau, bias, dtau, dbias)):
+        heads = ctypes.byref(solo_heads_t(_ptr(tau), _ptr(bias), _ptr(dtau), _ptr(dbias)))
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    st = load().solo_readout_fwd_bwd_private(
+        ctypes.byref(dims), arr(hidden), arr(gammas), arr(Ws), _ptr(targets), _ptr(mask), heads,
+        _ptr(loss_tok), _ptr(loss_mean), arr(dhidden), arr(dWs), arr(dgammas), _ptr(workspace),
+        int(workspace_bytes), _stream_handle(stream))
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd_private")
     return st
 
 

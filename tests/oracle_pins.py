@@ -442,3 +442,48 @@ def pin_heads_torch_fp64(orc):
 
 
 PINS += [pin_heads_finite_differences, pin_heads_closed_forms, pin_heads_torch_fp64]
+
+
+# -- private readouts -----------------------------------------------------------
+
+def pin_private_readouts(orc):
+    """With every W_k = W and gamma_k = gamma the private readouts reduce to the
+    shared one (losses, dH, and the final module's dW, dgamma); a module's own
+    dW_k and dgamma_k match central differences of its own loss."""
+    p = problem(K=3, N=5, d=8, V=12, seed=33, mask_frac=0.2, row_scale=True, orc=orc)
+    p["W"] = p["W"] * 15.0
+    K = p["K"]
+    shared = run(orc, p, contract=True)
+    priv = orc.solo_readout_private(p["hidden"], [p["gamma"]] * K, [p["W"]] * K, p["targets"],
+                                    eps=p["eps"], contract=True)
+    np.testing.assert_allclose(priv["loss_tok"], shared["loss_tok"], rtol=0, atol=1e-14)
+    for k in range(K):
+        assert rel(priv["dhidden"][k], shared["dhidden"][k]) < 1e-13
+    assert rel(priv["dW"][-1], shared["dW"]) < 1e-13
+    assert rel(priv["dgamma"][-1], shared["dgamma"]) < 1e-13
+    # distinct readouts: FD of module 0's loss in its own W_0 and gamma_0
+    rng = np.random.default_rng(4)
+    Ws = [p["W"] * (1.0 + 0.3 * rng.standard_normal(p["W"].shape)) for _ in range(K)]
+    gs = [p["gamma"] * (1.0 + 0.2 * rng.standard_normal(p["d"])) for _ in range(K)]
+    out = orc.solo_readout_private(p["hidden"], gs, Ws, p["targets"], eps=p["eps"],
+                                   contract=False)
+    step = 1e-6
+    L0 = lambda W0, g0: orc.solo_readout_private(p["hidden"][:1], [g0], [W0], p["targets"][:1],
+                                                 eps=p["eps"], contract=False)["loss_mean"][0]
+    numW = np.zeros_like(Ws[0])
+    for idx in np.ndindex(*numW.shape):
+        Wp, Wm = Ws[0].copy(), Ws[0].copy()
+        Wp[idx] += step
+        Wm[idx] -= step
+        numW[idx] = (L0(Wp, gs[0]) - L0(Wm, gs[0])) / (2 * step)
+    assert rel(out["dW"][0], numW) < 1e-7
+    numg = np.zeros(p["d"])
+    for j in range(p["d"]):
+        gp, gm = gs[0].copy(), gs[0].copy()
+        gp[j] += step
+        gm[j] -= step
+        numg[j] = (L0(Ws[0], gp) - L0(Ws[0], gm)) / (2 * step)
+    assert rel(out["dgamma"][0], numg) < 1e-7
+
+
+PINS.append(pin_private_readouts)

@@ -148,3 +148,17 @@ def test_exit_readout_host_checks(sr):
     assert sr.solo_readout_exit_forward(dims, [fake, fake], fake, fake, fake, None, None, None,
                                         fake, None, fake, workspace_bytes=small - 1, stream=0,
                                         check=False) == sr.SOLO_ERR_WORKSPACE_TOO_SMALL
+
+
+def test_private_host_checks(sr):
+    fake = 1 << 20
+    dims = sr.make_dims(3, 64, 64, 100)
+    one = sr.solo_readout_private_workspace_bytes(dims)
+    assert one < sr.solo_readout_workspace_bytes(dims)
+    args = dict(hidden=[fake] * 3, gammas=[fake] * 3, Ws=[fake, fake, fake], targets=fake,
+                mask=None, loss_tok=None, loss_mean=fake, dhidden=[fake] * 3, dWs=None,
+                dgammas=None, workspace=fake, stream=0, check=False)
+    assert sr.solo_readout_fwd_bwd_private(dims, **dict(args, Ws=[fake, None, fake]),
+                                           workspace_bytes=one) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_fwd_bwd_private(dims, **args, workspace_bytes=one - 1) == \
+        sr.SOLO_ERR_WORKSPACE_TOO_SMALL
