@@ -36,6 +36,8 @@
 //
 // Every wait is bounded (ptx.cuh); on a timeout all roles unwind, in-flight
 // copies and MMAs are drained, TMEM is freed and SOLO_FLAG_TIMEOUT is set.
+#include <algorithm>
+
 #include "internal.h"
 #include "ptx.cuh"
 #include "../../include/solo_readout.h"
@@ -74,6 +76,24 @@ __device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, i
   nb = r / gm;
 }
 
+// Work unit u -> tile, part of the tile (0 for a whole tile) and its
+// reduction blocks [kb_lo, kb_hi).
+__device__ __forceinline__ void unit_range(int u, const GemmArgs& a, int& t, int& part,
+                                           int& kb_lo, int& kb_hi) {
+  if (u < a.full_tiles) {
+    t = u;
+    part = 0;
+    kb_lo = 0;
+    kb_hi = a.k_blocks;
+    return;
+  }
+  const int i = u - a.full_tiles;
+  t = a.full_tiles + i / a.split;
+  part = i % a.split;
+  kb_lo = static_cast<int>(static_cast<int64_t>(part) * a.k_blocks / a.split);
+  kb_hi = static_cast<int>(static_cast<int64_t>(part + 1) * a.k_blocks / a.split);
+}
+
 // Waits without looking at the abort flag, bounded in time: used to drain
 // copies and MMAs that were already issued when a role gave up.
 __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
@@ -92,7 +112,8 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
 template <int MODE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const __grid_constant__ CUtensorMap tmD, const GemmArgs args) {
+                const __grid_constant__ CUtensorMap tmD, const __grid_constant__ CUtensorMap tmX,
+                const GemmArgs args) {
   constexpr bool kAmn = (MODE == kDW);
   constexpr bool kBmn = (MODE == kDxhat || MODE == kDW);
   constexpr uint32_t kIdesc = idesc_bf16_f32(kPairRows, kBN, kAmn, kBmn);
@@ -149,12 +170,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       uint32_t stage = 0, phase = 0;
       uint32_t issued = 0, last_phase = 0;   // per-stage bits for draining
       bool ok = true;
-      for (int t = cluster; ok && t < args.num_tiles; t += num_clusters) {
-        int mb, nb;
+      for (int u = cluster; ok && u < args.num_units; u += num_clusters) {
+        int t, part, kb_lo, kb_hi, mb, nb;
+        unit_range(u, args, t, part, kb_lo, kb_hi);
         tile_coords(t, args, mb, nb);
         const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
         const int n0 = nb * kBN + static_cast<int>(rank) * kBHalf;
-        for (int kb = 0; kb < args.k_blocks; ++kb) {
+        for (int kb = kb_lo; kb < kb_hi; ++kb) {
           if (!mbar_wait_cluster(&empty[stage], phase ^ 1, abort_flag)) {
             ok = false;
             break;
@@ -217,7 +239,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       bool ok = true;
       const uint32_t a_base = smem_u32(smem + kSmemA);
       const uint32_t b_base = smem_u32(smem + kSmemB);
-      for (int t = cluster; ok && t < args.num_tiles; t += num_clusters, ++local) {
+      for (int u = cluster; ok && u < args.num_units; u += num_clusters, ++local) {
+        int t, part, kb_lo, kb_hi;
+        unit_range(u, args, t, part, kb_lo, kb_hi);
         const uint32_t acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait_cluster(&tempty[acc], acc_phase ^ 1, abort_flag)) {
@@ -226,7 +250,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * kBN;
-        for (int kb = 0; kb < args.k_blocks; ++kb) {
+        for (int kb = kb_lo; kb < kb_hi; ++kb) {
           if (!mbar_wait_cluster(&full[stage], phase, abort_flag)) {
             ok = false;
             break;
@@ -240,7 +264,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                                      : smem_desc_sw128(sa + k * 32, 16, 1024);
             const uint64_t bd = kBmn ? smem_desc_sw128(sb + k * 2048, 8192, 1024)
                                      : smem_desc_sw128(sb + k * 32, 16, 1024);
-            mma_bf16_pair(d_tmem, ad, bd, kIdesc, (kb | k) != 0 ? 1u : 0u);
+            mma_bf16_pair(d_tmem, ad, bd, kIdesc, (kb != kb_lo || k != 0) ? 1u : 0u);
           }
           mma_commit_pair(&empty[stage], kBothCtas);
           if (++stage == kStages) {
@@ -267,8 +291,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     int buf = 0;
     int local = 0;
     bool ok = true;
-    for (int t = cluster; t < args.num_tiles; t += num_clusters, ++local) {
-      int mb, nb;
+    for (int u = cluster; u < args.num_units; u += num_clusters, ++local) {
+      int t, part, kb_lo, kb_hi, mb, nb;
+      unit_range(u, args, t, part, kb_lo, kb_hi);
       tile_coords(t, args, mb, nb);
       const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
       const int n0 = nb * kBN;
@@ -451,7 +476,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
+            if (part == 0) {
+              tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
+            } else {    // a later reduction range of a cut tile: its auxiliary slot
+              const int slot = (t - args.full_tiles) * (args.split - 1) + part - 1;
+              tma_store_2d(&tmX, ebuf + buf * kEpiBufBytes, c * 32,
+                           slot * kPairRows + static_cast<int>(rank) * kBM + 32 * q);
+            }
             bulk_commit_group();
           }
           buf ^= 1;
@@ -497,27 +528,84 @@ cudaError_t gemm_prepare(int /*device*/) {
   return e;
 }
 
+void plan_units(GemmArgs& g, int sms, bool allow_split) {
+  g.full_tiles = g.num_tiles;
+  g.split = 1;
+  g.num_units = g.num_tiles;
+  const int pairs = std::min(std::max(sms / 2, 1), kMaxAuxSlots + 1);
+  const int rem = g.num_tiles % pairs;
+  if (!allow_split || rem == 0) return;
+  int s = std::min({pairs / rem, kMaxSplit, g.k_blocks});
+  while (s > 1 && rem * (s - 1) > kMaxAuxSlots) --s;
+  if (s < 2) return;
+  g.full_tiles = g.num_tiles - rem;
+  g.split = s;
+  g.num_units = g.full_tiles + rem * s;
+}
+
+namespace {
+
+// out[tile] += aux parts 1 .. split-1 of each cut tile, in that order.
+// Grid (cut tiles, 256 / 16 row chunks), 256 threads: 16 rows x 64 float4.
+__global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, float* out,
+                                                          int64_t ld, const float* aux) {
+  const int cut = blockIdx.x;
+  const int t = g.full_tiles + cut;
+  int mb, nb;
+  tile_coords(t, g, mb, nb);
+  const int lr = blockIdx.y * 16 + (threadIdx.x >> 6);     // row within the tile (+ 4 x 4)
+  const int c4 = threadIdx.x & 63;                          // float4 column within the tile
+  const int col = nb * kBN + 4 * c4;
+  for (int rr = 0; rr < 16; rr += 4) {
+    const int r = lr + rr;
+    const int64_t row = static_cast<int64_t>(mb) * kPairRows + r;
+    if (row >= g.M || col >= g.N) continue;        // N is a multiple of 8: whole float4s
+    float4* o = reinterpret_cast<float4*>(out + row * ld + col);
+    float4 acc = *o;
+    for (int p = 1; p < g.split; ++p) {
+      const int slot = cut * (g.split - 1) + p - 1;
+      const float4 x = *reinterpret_cast<const float4*>(
+          aux + (static_cast<int64_t>(slot) * kPairRows + r) * kBN + 4 * c4);
+      acc.x += x.x;
+      acc.y += x.y;
+      acc.z += x.z;
+      acc.w += x.w;
+    }
+    *o = acc;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const float* aux,
+                               cudaStream_t stream) {
+  const int cut = g.num_tiles - g.full_tiles;
+  if (g.split < 2 || cut <= 0) return cudaSuccess;
+  split_fixup_kernel<<<dim3(cut, kPairRows / 16), 256, 0, stream>>>(g, out, ld, aux);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
-                        const CUtensorMap& d, const GemmArgs& args, int sms,
-                        cudaStream_t stream) {
-  if (args.num_tiles <= 0) return cudaSuccess;
-  const int clusters = std::min(args.num_tiles, std::max(sms / 2, 1));
+                        const CUtensorMap& d, const CUtensorMap& x, const GemmArgs& args,
+                        int sms, cudaStream_t stream) {
+  if (args.num_units <= 0) return cudaSuccess;
+  const int clusters = std::min(args.num_units, std::max(sms / 2, 1));
   const int grid = 2 * clusters;
   switch (mode) {
     case kLogits:
-      gemm_kernel<kLogits><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      gemm_kernel<kLogits><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
     case kDxhat:
-      gemm_kernel<kDxhat><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      gemm_kernel<kDxhat><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
     case kDW:
-      gemm_kernel<kDW><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      gemm_kernel<kDW><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
     case kExit:
-      gemm_kernel<kExit><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      gemm_kernel<kExit><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
     case kLogitsHeads:
-      gemm_kernel<kLogitsHeads><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, args);
+      gemm_kernel<kLogitsHeads><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
   }
   return cudaGetLastError();

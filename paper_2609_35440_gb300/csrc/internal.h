@@ -38,6 +38,14 @@ struct GemmArgs {
   int32_t n_blocks;   // 256-column blocks
   int32_t group_m;    // tile raster: group_m row blocks sweep all column blocks together
   int32_t num_tiles;
+  // Work units: tiles [0, full_tiles) whole, then each remaining tile cut
+  // into `split` contiguous reduction ranges (fills the last partial wave of
+  // CTA pairs).  Part 0 of a cut tile is stored to the output, parts 1.. to
+  // the auxiliary buffer (slot (tile - full_tiles) * (split - 1) + part - 1,
+  // 256 x 256 fp32 each) and added by launch_split_fixup in a fixed order.
+  int32_t full_tiles;
+  int32_t split;
+  int32_t num_units;
   // kLogits epilogue
   const int32_t* targets;  // [M] token targets (flattened [K, N])
   float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile
@@ -55,10 +63,29 @@ struct GemmArgs {
 
 size_t gemm_smem_bytes();
 cudaError_t gemm_prepare(int device);  // sets the dynamic shared memory limit once per device
-// Launches min(tiles, sms / 2) CTA pairs.
+
+constexpr int kMaxSplit = 8;        // reduction ranges per cut tile
+constexpr int kMaxAuxSlots = 127;   // 256 x 256 fp32 partial tiles (32 MB)
+// Auxiliary slots a product of `tiles` tiles and `k_blocks` reduction blocks
+// may need (a part keeps at least one reduction block).
+inline int split_aux_slots(int64_t tiles, int64_t k_blocks) {
+  const int64_t parts = k_blocks < kMaxSplit ? k_blocks : kMaxSplit;
+  const int64_t s = tiles * (parts - 1);
+  return static_cast<int>(s < kMaxAuxSlots ? s : kMaxAuxSlots);
+}
+// Sets full_tiles / split / num_units: whole tiles fill complete waves of
+// min(sms / 2, kMaxAuxSlots + 1) pairs; the remainder is cut so the last wave
+// has as many units as pairs (each part keeps >= 1 reduction block).
+// allow_split = false keeps every tile whole.
+void plan_units(GemmArgs& g, int sms, bool allow_split);
+// Launches min(units, sms / 2) CTA pairs.  x: tensor map of the auxiliary
+// buffer (fp32 [slots * 256, 256], 32 x 32 boxes) for the cut tiles' parts.
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
-                        const CUtensorMap& d, const GemmArgs& args, int sms,
-                        cudaStream_t stream);
+                        const CUtensorMap& d, const CUtensorMap& x, const GemmArgs& args,
+                        int sms, cudaStream_t stream);
+// out (fp32, row stride ld) += the auxiliary parts of every cut tile.
+cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const float* aux,
+                               cudaStream_t stream);
 
 // ---- row kernels ---------------------------------------------------------------
 

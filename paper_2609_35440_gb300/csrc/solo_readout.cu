@@ -13,6 +13,7 @@
 //   dgamma       fixed-order sum of the partials                  [d]
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -42,7 +43,8 @@ struct Layout {
   int db_chunks = 0;
   size_t flags = 0, r = 0, lse = 0, zy = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
   size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0;
-  size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, total = 0;
+  size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
+  int aux_slots = 0;
 };
 
 solo_status_t check_dims(const solo_dims_t* d) {
@@ -90,6 +92,13 @@ Layout make_layout(const solo_dims_t& d) {
   L.sy = take(M * 4);
   L.part_tau = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
   L.db_part = take(static_cast<size_t>(d.K) * L.db_chunks * L.ldp * 4);
+  // partial tiles of the dX̂ and dW products' last wave (one at a time)
+  const int64_t nb = (d.d + kBN - 1) / kBN;
+  const int64_t tiles_dx = (L.M + 2 * kBM - 1) / (2 * kBM) * nb;
+  const int64_t tiles_dw = (d.V + 2 * kBM - 1) / (2 * kBM) * nb;
+  L.aux_slots = std::max(split_aux_slots(tiles_dx, (d.V + kBK - 1) / kBK),
+                         split_aux_slots(tiles_dw, (d.N + kBK - 1) / kBK));
+  L.aux = take(static_cast<size_t>(std::max(L.aux_slots, 1)) * 2 * kBM * kBN * 4);
   L.total = off;
   return L;
 }
@@ -251,8 +260,12 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   const uint64_t V = static_cast<uint64_t>(D.V);
   const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
-  CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW;
+  CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW, mAux;
+  float* aux = reinterpret_cast<float*>(ws + L.aux);
   bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, kBK, kBM) &&
+            make_map(&mAux, F32, aux, kBN,
+                     static_cast<uint64_t>(std::max(L.aux_slots, 1)) * 2 * kBM, kBN * 4, 32,
+                     32) &&
             make_map(&mW_k, BF, W, d, V, d * 2, kBK, kBN / 2) &&
             make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
             make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, kBK, kBM) &&
@@ -295,8 +308,10 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.tokens_per_module = D.N;
   g.usum = ra.usum;
   g.sy = ra.sy;
+  plan_units(g, sms, false);
   if (!mark(SOLO_STAGE_LOGITS) ||
-      fail(launch_gemm(affine ? kLogitsHeads : kLogits, mX_k, mW_k, mP_st, g, sms, stream)))
+      fail(launch_gemm(affine ? kLogitsHeads : kLogits, mX_k, mW_k, mP_st, mAux, g, sms,
+                       stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_LSE) || fail(launch_lse(ra, stream, dtau != nullptr)))
@@ -309,8 +324,10 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
   gx.group_m = kGroupDxhat;
   gx.num_tiles = gx.m_blocks * gx.n_blocks;
+  plan_units(gx, sms, true);
   if (!mark(SOLO_STAGE_DXHAT) ||
-      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, gx, sms, stream)))
+      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, mAux, gx, sms, stream)) ||
+      fail(launch_split_fixup(gx, ra.dxhat, D.d, aux, stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_norm_bwd(ra, stream, dgamma != nullptr)))
@@ -327,7 +344,9 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
     gw.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
     gw.group_m = kGroupDW;
     gw.num_tiles = gw.m_blocks * gw.n_blocks;
-    if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, gw, sms, stream)))
+    plan_units(gw, sms, true);
+    if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, mAux, gw, sms, stream)) ||
+        fail(launch_split_fixup(gw, dW, D.d, aux, stream)))
       return SOLO_ERR_CUDA;
   }
   if (!mark(SOLO_STAGE_DGAMMA)) return SOLO_ERR_CUDA;
@@ -449,6 +468,7 @@ solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden
   g.n_blocks = L.n_tiles_v;
   g.group_m = kGroupLogits;
   g.num_tiles = g.m_blocks * g.n_blocks;
+  plan_units(g, sms, false);
   g.targets = targets;
   g.stats = ra.stats;
   g.zy = ra.zy;
@@ -456,7 +476,7 @@ solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden
   g.flags = ra.flags;
   g.argmax = ra.argmax;
   // the store map is unused by this epilogue; any valid map fills the slot
-  if (!mark(1) || launch_gemm(kExit, mX_k, mW_k, mX_k, g, sms, stream) != cudaSuccess)
+  if (!mark(1) || launch_gemm(kExit, mX_k, mW_k, mX_k, mX_k, g, sms, stream) != cudaSuccess)
     return SOLO_ERR_CUDA;
   if (!mark(2) || launch_exit_lse(ra, stream) != cudaSuccess) return SOLO_ERR_CUDA;
   if (!mark(3)) return SOLO_ERR_CUDA;
