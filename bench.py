@@ -391,10 +391,12 @@ def run_ours(args, wl):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     barrier()
+    launches0 = sr.solo_readout_kernel_launches()
     t0.record(stream)
     for i in range(args.steps):
         ro(hidden, gamma, W, targets, stream=stream, events=step_evs[i], **heads)
     t1.record(stream)
+    launches = sr.solo_readout_kernel_launches() - launches0
     barrier()
     clk.__exit__(None, None, None)
     flags = ro.flags(stream)
@@ -454,9 +456,6 @@ def run_ours(args, wl):
     cpu = None
     if not args.no_cpu:
         cpu = cpu_baseline(wl, args.cpu_seconds)
-    # rmsnorm, logits, lse + module means, grad, dxhat, norm_bwd, dgamma parts, dW, dgamma
-    # (+ the bias-gradient reduction with heads)
-    launches_per_step = 11 if heads else 10
     line = {
         "metric": HEADS_METRIC if heads else METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": world,
@@ -478,7 +477,7 @@ def run_ours(args, wl):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "clocks": clk.summary(),
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": launches,       # the library's own count over the timed calls
         "device_flags": flags,
     }
     print(json.dumps(line), flush=True)
@@ -524,10 +523,12 @@ def run_exit_bench(args, wl):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize(dev)
+    launches0 = sr.solo_readout_kernel_launches()
     t0.record(stream)
     for i in range(args.steps):
         ex(hidden, gamma, W, targets, stream=stream, events=evs[i])
     t1.record(stream)
+    launches = sr.solo_readout_kernel_launches() - launches0
     torch.cuda.synchronize(dev)
     clk.__exit__(None, None, None)
     ms = t0.elapsed_time(t1)
@@ -591,7 +592,7 @@ def run_exit_bench(args, wl):
                 "h2d_bytes_per_step": sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4,
                 "d2h_bytes_per_step": lt_host.numel() * 4 + top_host.numel() * 4},
         "clocks": clk.summary(),
-        "gpu_launches": 4 * args.steps,   # rmsnorm, exit GEMM, combine, module means
+        "gpu_launches": launches,       # the library's own count over the timed calls
         "device_flags": flags,
     }
     print(json.dumps(line), flush=True)
@@ -630,10 +631,12 @@ def run_private_bench(args, wl):
     torch.cuda.synchronize(dev)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    launches0 = sr.solo_readout_kernel_launches()
     t0.record(stream)
     for _ in range(args.steps):
         call()
     t1.record(stream)
+    launches = sr.solo_readout_kernel_launches() - launches0
     torch.cuda.synchronize(dev)
     clk.__exit__(None, None, None)
     ms = t0.elapsed_time(t1)
@@ -650,7 +653,7 @@ def run_private_bench(args, wl):
             "algo_tflops": tflops,
             "algo_frac_of_peak": tflops / peak,
             "peak_source": f"{peak_src} bf16_tflops_sustained",
-            "clocks": clk.summary(), "gpu_launches": 10 * K * args.steps,
+            "clocks": clk.summary(), "gpu_launches": launches,
             "device_flags": sr.solo_readout_get_flags(ws, stream)}
     print(json.dumps(line), flush=True)
 

@@ -326,6 +326,15 @@ solo_status_t solo_readout_selftest_wait_timeout(uint32_t* device_flags, uint32_
 int32_t solo_readout_version(void);
 
 /*
+ * Number of kernels this library has enqueued in the calling process so far
+ * (all threads, all devices; each successful launch counts once).  A
+ * caller that reads it before and after a sequence of calls gets the exact
+ * number of the library's kernels in that sequence.  Host-only and
+ * lock-free; it does not synchronise with the device.
+ */
+uint64_t solo_readout_kernel_launches(void);
+
+/*
  * Size of the library's built-in scratch area used by
  * solo_readout_fwd_bwd_static: 64 MiB of device memory, reserved on every GPU
  * that loads the library's device code and held until the process exits.

@@ -582,7 +582,7 @@ cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const 
   const int cut = g.num_tiles - g.full_tiles;
   if (g.split < 2 || cut <= 0) return cudaSuccess;
   split_fixup_kernel<<<dim3(cut, kPairRows / 16), 256, 0, stream>>>(g, out, ld, aux);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
@@ -608,7 +608,7 @@ cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& 
       gemm_kernel<kLogitsHeads><<<grid, kGemmThreads, kSmemTotal, stream>>>(a, b, d, x, args);
       break;
   }
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace solo

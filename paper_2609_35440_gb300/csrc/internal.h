@@ -7,6 +7,17 @@
 
 namespace solo {
 
+// Every kernel launch of the library goes through launched(): it returns the
+// launch's error and counts the successful ones for
+// solo_readout_kernel_launches.
+void note_launch();
+uint64_t launch_count();
+inline cudaError_t launched() {
+  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) note_launch();
+  return e;
+}
+
 // Tensor-core tile: a CTA pair computes 256 rows x 256 columns (each CTA owns
 // 128 rows), reduction in blocks of 64 through a 6-stage shared-memory ring.
 constexpr int kBM = 128;

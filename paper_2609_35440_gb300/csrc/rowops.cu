@@ -559,7 +559,7 @@ cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
     case 8: rmsnorm_fwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
     default: rmsnorm_fwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
   }
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads) {
@@ -567,28 +567,28 @@ cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads) {
     lse_kernel<kLseHeads><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
   else
     lse_kernel<kLseTrain><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launched();
   if (e != cudaSuccess) return e;
   module_mean_kernel<<<a.K, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s) {
   lse_kernel<kLseExit><<<dim3(a.part_blocks, a.K), 256, 0, s>>>(a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launched();
   if (e != cudaSuccess) return e;
   module_mean_kernel<<<a.K, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
   if (a.dbias) {
     const dim3 grid((a.ldp / 8 + 255) / 256, a.K * a.db_chunks);
     grad_colsum_kernel<<<grid, 256, 0, s>>>(a);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launched();
     if (e != cudaSuccess) return e;
     dbias_reduce_kernel<<<dim3((a.V + 255) / 256, a.K), 256, 0, s>>>(a);
-    return cudaGetLastError();
+    return launched();
   }
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const size_t smem = static_cast<size_t>(a.n_tiles_v) * sizeof(float);
@@ -599,7 +599,7 @@ cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
     if (e != cudaSuccess) return e;
   }
   grad_rows_kernel<<<static_cast<unsigned>(M), 256, smem, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts) {
@@ -612,15 +612,15 @@ cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_p
     case 8: norm_bwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
     default: norm_bwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
   }
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launched();
   if (e != cudaSuccess || !want_dgamma_parts) return e;
   dgamma_part_kernel<<<dim3((a.d + 255) / 256, a.dg_chunks), 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s) {
   dgamma_reduce_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace solo

@@ -35,5 +35,5 @@ extern "C" solo_status_t solo_readout_selftest_wait_timeout(uint32_t* device_fla
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   solo::wait_timeout_selftest_kernel<<<1, 32, 0, s>>>(device_flags,
                                                       static_cast<uint64_t>(limit_us) * 1000ull);
-  return cudaGetLastError() == cudaSuccess ? SOLO_OK : SOLO_ERR_CUDA;
+  return solo::launched() == cudaSuccess ? SOLO_OK : SOLO_ERR_CUDA;
 }

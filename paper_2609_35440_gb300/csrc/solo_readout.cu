@@ -14,12 +14,24 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <mutex>
 
 #include "../../include/solo_readout.h"
 #include "internal.h"
+
+namespace solo {
+
+namespace {
+std::atomic<uint64_t> g_launches{0};
+}  // namespace
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+uint64_t launch_count() { return g_launches.load(std::memory_order_relaxed); }
+
+}  // namespace solo
 
 namespace {
 
@@ -646,6 +658,8 @@ const char* solo_readout_strerror(solo_status_t status) {
 }
 
 int32_t solo_readout_version(void) { return 100; }
+
+uint64_t solo_readout_kernel_launches(void) { return solo::launch_count(); }
 
 }  // extern "C"
 

@@ -109,6 +109,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_fwd_bwd_private.restype = i32
     lib.solo_readout_version.argtypes = []
     lib.solo_readout_version.restype = i32
+    lib.solo_readout_kernel_launches.argtypes = []
+    lib.solo_readout_kernel_launches.restype = ctypes.c_uint64
     _lib = lib
     return lib
 
@@ -348,6 +350,11 @@ def solo_readout_selftest_wait_timeout(device_flags, limit_us: int, stream=None,
 
 def solo_readout_version() -> int:
     return load().solo_readout_version()
+
+
+def solo_readout_kernel_launches() -> int:
+    """Kernels the library has enqueued in this process so far."""
+    return int(load().solo_readout_kernel_launches())
 
 
 class Readout:

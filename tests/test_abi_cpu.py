@@ -162,3 +162,14 @@ def test_private_host_checks(sr):
                                            workspace_bytes=one) == sr.SOLO_ERR_INVALID_ARG
     assert sr.solo_readout_fwd_bwd_private(dims, **args, workspace_bytes=one - 1) == \
         sr.SOLO_ERR_WORKSPACE_TOO_SMALL
+
+
+def test_launch_counter_ignores_rejected_calls(sr):
+    """Calls refused on the host enqueue nothing, so the counter stays put."""
+    before = sr.solo_readout_kernel_launches()
+    a = _args(sr, workspace_bytes=1024)
+    assert sr.solo_readout_fwd_bwd(a["dims"], a["hidden"], a["gamma"], a["W"], a["targets"],
+                                   None, None, a["loss_mean"], a["dhidden"], None, None,
+                                   a["workspace"], workspace_bytes=1024, stream=0,
+                                   check=False) == sr.SOLO_ERR_WORKSPACE_TOO_SMALL
+    assert sr.solo_readout_kernel_launches() == before

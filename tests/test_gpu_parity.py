@@ -122,3 +122,32 @@ def test_workspace_reuse_across_shapes():
            torch.from_numpy(inp.targets).cuda())
         torch.cuda.synchronize()
         assert torch.equal(ro.loss_mean.cpu(), torch.from_numpy(gpu["loss_mean"]).float())
+
+
+def test_kernel_launch_counter():
+    """The library's launch counter sees every kernel of a call: the same call
+    twice counts the same, the split last wave adds its fix-up kernels, and
+    leaving out dW and dgamma removes their kernels."""
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    wl = Workload("k2_n600_d256_v3000", K=2, N=600, d=256, V=3000, seed=46)
+    inp = synth.generate(wl)
+    hid = [parity.to_device_bf16(inp.hidden[k]) for k in range(wl.K)]
+    gamma, W = parity.to_device_bf16(inp.gamma), parity.to_device_bf16(inp.W)
+    tg = torch.from_numpy(inp.targets).cuda()
+
+    def count(**kw):
+        ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, **kw)
+        n0 = sr.solo_readout_kernel_launches()
+        ro(hid, gamma, W, tg)
+        n = sr.solo_readout_kernel_launches() - n0
+        torch.cuda.synchronize()
+        return n
+
+    full = count()
+    assert full == count()
+    # rmsnorm, logits, lse, module means, grad, dxhat, norm_bwd, dgamma parts, dW,
+    # dgamma reduce: 10, plus one fix-up per product whose last wave was cut
+    assert 10 <= full <= 12
+    # without dW and dgamma: no dW GEMM (nor its fix-up), dgamma parts or reduction
+    assert 7 <= count(want_dW=False, want_dgamma=False) <= full - 3
