@@ -1,4 +1,4 @@
-// Persistent tcgen05 GEMM for sm_103a on CTA pairs, with three fused epilogues.
+// Persistent tcgen05 GEMM for sm_103a on CTA pairs, with five epilogue modes.
 //
 // Two CTAs on neighbouring SMs form a cluster and compute one 256 x 256
 // output tile together with tcgen05.mma.cta_group::2 (M = 256, N = 256, K =
@@ -16,6 +16,12 @@
 //   warps 2-5  epilogue: each owns 32 TMEM lanes (rows) of its CTA's 128
 //              rows x 256 columns; releases the accumulator on the even CTA's
 //              "tmem empty" barrier (8 arrivals: 4 warps x 2 CTAs)
+//
+// Work units: the pairs take units round robin.  A unit is a whole tile, or,
+// for the tiles that do not fill a last complete wave of pairs (kDxhat, kDW),
+// one of up to 8 contiguous ranges of the tile's reduction; part 0 of such a
+// tile is stored to the output and the other parts to auxiliary slots that
+// launch_split_fixup adds back in a fixed order.
 //
 // Epilogues:
 //  kLogits  Z = Xhat W^T.  Per row and 256-column tile: m = max_v z,

@@ -46,6 +46,10 @@ RAGGED = [
     Workload("k2_n1_d8_v16", K=2, N=1, d=8, V=16, seed=35),
     Workload("k2_n300_d512_v2500_heavy", K=2, N=300, d=512, V=2500, seed=36, heavy_frac=0.01,
              row_scale=True, mask_frac=0.05),
+    # the largest module count the call takes (SOLO_MAX_MODULES)
+    Workload("k16_n40_d64_v777", K=16, N=40, d=64, V=777, seed=37, mask_frac=0.05),
+    # d above 2048: the row kernels' generic path (rows re-read instead of cached)
+    Workload("k2_n70_d2600_v600", K=2, N=70, d=2600, V=600, seed=38, row_scale=True),
 ]
 
 
