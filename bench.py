@@ -91,11 +91,22 @@ def load_peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
+def strip_comments(src: str) -> str:
+    """C++ source without comments, blank lines or trailing spaces (string
+    literals in these files hold no comment markers)."""
+    import re
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    return "\n".join(ln.rstrip() for ln in src.splitlines() if ln.strip())
+
+
 def kernel_hash() -> str:
+    """Hash of the GEMM kernel's code (comments ignored): a committed traffic
+    capture applies only while this is unchanged."""
     h = hashlib.sha256()
     for rel in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, rel), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, rel), encoding="utf-8") as f:
+            h.update(strip_comments(f.read()).encode())
     return h.hexdigest()[:16]
 
 
