@@ -136,7 +136,7 @@ class ClockSampler:
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
-        self.index = index
+        self.index = 0 if index is None else index
         self.proc = None
         self.lines = []
 
@@ -511,7 +511,7 @@ def run_exit_bench(args, wl):
     from paper_2609_35440_gb300 import build
     build.ensure_built()
     sr.load()
-    dev = torch.device("cuda")
+    dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream(dev)
     inp = synth.generate(wl)
     to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
@@ -616,7 +616,7 @@ def run_private_bench(args, wl):
     from paper_2609_35440_gb300 import build
     build.ensure_built()
     sr.load()
-    dev = torch.device("cuda")
+    dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream(dev)
     inp = synth.generate(wl)
     to_dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(
