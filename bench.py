@@ -215,6 +215,11 @@ def replica_workload(wl, rank: int):
 
 # ----------------------------------------------------------------------- e2e
 
+E2E_METHOD = ("every step: its hidden states and targets copied from pinned host memory "
+              "into one of two device buffers on a copy stream (overlapping the previous "
+              "step's compute), the call, and its losses copied back; all inside the timed "
+              "region")
+
 def pipelined_e2e(torch, dev, stream, h_host, t_host, hidden, targets, compute, read_back,
                   steps, warm=2):
     """Times `steps` end-to-end steps: each step's inputs are copied from pinned host
@@ -446,7 +451,7 @@ def run_ours(args, wl):
         h2d = sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4
         d2h = lt_host.numel() * 4 + lm_host.numel() * 4
         e2e = {"value": job_throughput(tokens_step, steps_e2e, world, ems), "unit": "tokens/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "method": E2E_METHOD}
 
     if rank != 0:
         if world > 1:
@@ -601,7 +606,8 @@ def run_exit_bench(args, wl):
         "cpu_baseline": cpu,
         "e2e": {"value": job_throughput(wl.M, steps_e2e, 1, ems), "unit": "tokens/s",
                 "h2d_bytes_per_step": sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4,
-                "d2h_bytes_per_step": lt_host.numel() * 4 + top_host.numel() * 4},
+                "d2h_bytes_per_step": lt_host.numel() * 4 + top_host.numel() * 4,
+                "method": E2E_METHOD.replace("its losses", "its losses and top-1")},
         "clocks": clk.summary(),
         "gpu_launches": launches,       # the library's own count over the timed calls
         "device_flags": flags,
