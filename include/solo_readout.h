@@ -20,7 +20,8 @@
  * Conventions for every entry point:
  *  - Pointers are DEVICE pointers unless the comment says "host".  The caller
  *    owns all memory; the library allocates nothing and keeps no state
- *    between calls besides per-device kernel attributes set on first use.
+ *    between calls besides per-device kernel attributes set on first use
+ *    and a process-wide count of the kernels it has launched.
  *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *    default stream).  Errors the host can detect are returned before any
  *    work is enqueued; conditions found on the device set bits of a flag
@@ -94,8 +95,8 @@ typedef struct {
 /*
  * Bytes of device workspace one call with these dims needs (host-only; no
  * CUDA call).  The workspace holds the normalised inputs, the bf16
- * exponentials/gradient of the logits ([K*N, V]), per-token statistics and
- * the flag word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims
+ * exponentials/gradient of the logits ([K*N, V]), per-token statistics,
+ * fp32 partial tiles of the backward products and the flag word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims
  * out of range, SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0.
  */
 solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
