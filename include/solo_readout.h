@@ -63,8 +63,12 @@ enum {
 enum {
   SOLO_FLAG_BAD_TARGET = 1u, /* a target outside [0, V) that is not ignore_index;
                                 the token is treated as masked */
-  SOLO_FLAG_TIMEOUT = 2u     /* a pipeline wait exceeded its bound (about 2 s);
+  SOLO_FLAG_TIMEOUT = 2u,    /* a pipeline wait exceeded its bound (about 2 s);
                                 the kernel stopped early and outputs are invalid */
+  SOLO_FLAG_BOUNDS = 4u      /* checked builds only (solo_readout_build_flags bit
+                                SOLO_BUILD_CHECKED): a computed global index fell
+                                outside its buffer; the access was skipped and
+                                outputs are invalid */
 };
 
 /* Maximum number of modules per call. */
@@ -325,6 +329,13 @@ solo_status_t solo_readout_selftest_wait_timeout(uint32_t* device_flags, uint32_
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 int32_t solo_readout_version(void);
+
+/* How the library was built: SOLO_BUILD_CHECKED is set in the checked build,
+ * whose kernels test every computed global index of the row kernels and the
+ * GEMM epilogues against its buffer and report SOLO_FLAG_BOUNDS instead of
+ * making the access.  Its results are bitwise those of the release build. */
+#define SOLO_BUILD_CHECKED 1
+int32_t solo_readout_build_flags(void);
 
 /*
  * Number of kernels this library has enqueued in the calling process so far

@@ -16,6 +16,9 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIBDIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIBDIR, "libsolo_readout.so")
+# The checked build: every computed global index of the row kernels and GEMM
+# epilogues is tested (SOLO_DEBUG=1); a violation sets SOLO_FLAG_BOUNDS.
+LIB_CHECKED = os.path.join(LIBDIR, "libsolo_readout_checked.so")
 SOURCES = ["gemm_tc.cu", "rowops.cu", "solo_readout.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
@@ -36,20 +39,28 @@ def _inputs() -> list[str]:
     return files
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(f) <= t for f in _inputs())
 
 
-def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
+def up_to_date_checked() -> bool:
+    return up_to_date(LIB_CHECKED)
+
+
+def build(verbose: bool = False, extra_flags: list[str] | None = None,
+          checked: bool = False) -> str:
+    """Compiles the release library (or, with checked=True, the checked one)."""
     os.makedirs(LIBDIR, exist_ok=True)
     cc = nvcc()
-    extra = list(extra_flags or [])
+    extra = list(extra_flags or []) + (["-DSOLO_DEBUG=1"] if checked else [])
+    target = LIB_CHECKED if checked else LIB
+    tag = "_checked" if checked else ""
     objs, procs = [], []
     for src in SOURCES:
-        obj = os.path.join(LIBDIR, src.replace(".cu", ".o"))
+        obj = os.path.join(LIBDIR, src.replace(".cu", tag + ".o"))
         cmd = [cc, *ARCH, *FLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             print(" ".join(cmd), flush=True)
@@ -64,13 +75,21 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
             failed.append(src)
     if failed:
         raise RuntimeError(f"nvcc failed on {failed}")
-    tmp = LIB + ".tmp"
+    tmp = target + ".tmp"
     cmd = [cc, *ARCH, "-shared", *objs, "-o", tmp]
     subprocess.run(cmd, check=True)
-    os.replace(tmp, LIB)
+    os.replace(tmp, target)
     for o in objs:
         os.remove(o)
-    return LIB
+    return target
+
+
+def build_all(verbose: bool = False) -> list[str]:
+    """The release and the checked library, compiled concurrently."""
+    from concurrent.futures import ThreadPoolExecutor
+    with ThreadPoolExecutor(2) as ex:
+        futs = [ex.submit(build, verbose, None, c) for c in (False, True)]
+        return [f.result() for f in futs]
 
 
 def ensure_built() -> str:

@@ -351,7 +351,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (even) mbar_arrive(&tempty[acc]);
           else mbar_arrive_remote(tempty_even + acc * 8);
         }
-        if (row_ok) {
+        if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
           args.argmax[static_cast<size_t>(nb) * args.M + row] = n0 + amax;
         }
@@ -368,7 +368,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         if constexpr (kHeads) {
           const int kmod = row_ok ? static_cast<int>(row / args.tokens_per_module) : 0;
           if (args.tau) tau = args.tau[kmod];
-          if (args.bias) brow = args.bias + static_cast<size_t>(kmod) * args.V + n0;
+          if (args.bias &&
+              in_bounds(kmod < args.M / args.tokens_per_module && n0 + ncols <= args.V,
+                        args.flags))
+            brow = args.bias + static_cast<size_t>(kmod) * args.V + n0;
         }
         // bias of one 32-column chunk; rows of a tile share their module, so a
         // warp's vector loads hit the same addresses
@@ -456,7 +459,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (even) mbar_arrive(&tempty[acc]);
           else mbar_arrive_remote(tempty_even + acc * 8);
         }
-        if (row_ok) {
+        if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
           if constexpr (kHeads) args.usum[static_cast<size_t>(nb) * args.M + row] = usum;
         }
@@ -486,8 +489,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
             } else {    // a later reduction range of a cut tile: its auxiliary slot
               const int slot = (t - args.full_tiles) * (args.split - 1) + part - 1;
-              tma_store_2d(&tmX, ebuf + buf * kEpiBufBytes, c * 32,
-                           slot * kPairRows + static_cast<int>(rank) * kBM + 32 * q);
+              if (in_bounds(slot >= 0 && slot < args.aux_slots, args.flags))
+                tma_store_2d(&tmX, ebuf + buf * kEpiBufBytes, c * 32,
+                             slot * kPairRows + static_cast<int>(rank) * kBM + 32 * q);
             }
             bulk_commit_group();
           }
@@ -570,6 +574,7 @@ __global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, floa
     float4 acc = *o;
     for (int p = 1; p < g.split; ++p) {
       const int slot = cut * (g.split - 1) + p - 1;
+      if (!in_bounds(slot < g.aux_slots, g.flags)) continue;
       const float4 x = *reinterpret_cast<const float4*>(
           aux + (static_cast<int64_t>(slot) * kPairRows + r) * kBN + 4 * c4);
       acc.x += x.x;

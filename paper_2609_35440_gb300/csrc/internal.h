@@ -5,7 +5,25 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#ifndef SOLO_DEBUG
+#define SOLO_DEBUG 0
+#endif
+
 namespace solo {
+
+// Checked builds (SOLO_DEBUG = 1) test computed global indices against the
+// extent of their buffer; a failed test sets SOLO_FLAG_BOUNDS (4) in the flag
+// word and the caller skips the access.  Release builds compile the tests away.
+__device__ __forceinline__ bool in_bounds(bool ok, uint32_t* flags) {
+#if SOLO_DEBUG
+  if (!ok) atomicOr(flags, 4u);
+  return ok;
+#else
+  (void)ok;
+  (void)flags;
+  return true;
+#endif
+}
 
 // Every kernel launch of the library goes through launched(): it returns the
 // launch's error and counts the successful ones for
@@ -57,6 +75,7 @@ struct GemmArgs {
   int32_t full_tiles;
   int32_t split;
   int32_t num_units;
+  int32_t aux_slots;       // slots in the auxiliary buffer
   // kLogits epilogue
   const int32_t* targets;  // [M] token targets (flattened [K, N])
   float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile

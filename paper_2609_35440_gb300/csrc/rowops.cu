@@ -238,7 +238,8 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     }
     const float l = mx + logf(s);
     if constexpr (kExit) {
-      if (a.top1) a.top1[row] = a.argmax[static_cast<int64_t>(best_tile) * M + row];
+      if (a.top1 && in_bounds(best_tile < a.n_tiles_v, a.flags))
+        a.top1[row] = a.argmax[static_cast<int64_t>(best_tile) * M + row];
       if (a.top1_logprob) a.top1_logprob[row] = mx - l;
     } else {
       a.lse[row] = l;
@@ -267,7 +268,8 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     stau[threadIdx.x >> 5] = tsum;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (threadIdx.x == 0 &&
+      in_bounds(k < a.K && static_cast<int>(blockIdx.x) < a.part_blocks, a.flags)) {
     double t = 0.0, tt = 0.0;
     int c = 0;
     for (int w = 0; w < 8; ++w) {
@@ -324,6 +326,7 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   extern __shared__ float ctile[];
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int64_t row = blockIdx.x;
+  if (!in_bounds(row < M, a.flags)) return;
   const int k = static_cast<int>(row / a.N);
   const int y = a.targets[row];
   uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
@@ -345,6 +348,7 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
       P[v] = make_uint4(0, 0, 0, 0);
       continue;
     }
+    if (!in_bounds(v0 / kBN < a.n_tiles_v, a.flags)) continue;
     const float c = ctile[v0 / kBN];
     float f[8];
     unpack8(P[v], f);
@@ -372,6 +376,7 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   const int64_t left = static_cast<int64_t>(k + 1) * a.N - row0;
   const int rows = left < kGradRows ? static_cast<int>(left) : kGradRows;
   const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
+  if (!in_bounds(k < a.K && row0 + rows <= M, a.flags)) return;
   const float w = a.inv_nvalid[k];
   const float tau = a.tau ? a.tau[k] : 1.f;
   if (threadIdx.x < rows) {
@@ -426,6 +431,7 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
           make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
     }
   }
+  if (!in_bounds(chunk < a.db_chunks && col0 + 8 <= a.ldp, a.flags)) return;
   float* out = a.db_part + (static_cast<int64_t>(k) * a.db_chunks + chunk) * a.ldp + col0;
   reinterpret_cast<float4*>(out)[0] = make_float4(colsum[0], colsum[1], colsum[2], colsum[3]);
   reinterpret_cast<float4*>(out)[1] = make_float4(colsum[4], colsum[5], colsum[6], colsum[7]);
@@ -523,6 +529,8 @@ __global__ void __launch_bounds__(256) dgamma_part_kernel(const RowArgs a) {
   const int64_t n1 = min(a.N, n0 + a.dg_rows);
   const uint16_t* h = a.hidden[k];
   const int64_t row0 = static_cast<int64_t>(k) * a.N;
+  if (!in_bounds(chunk < a.dg_chunks && row0 + n1 <= static_cast<int64_t>(a.K) * a.N, a.flags))
+    return;
   float acc = 0.f;
   for (int64_t n = n0; n < n1; ++n) {
     const float hv = __uint_as_float(static_cast<uint32_t>(h[n * a.d + j]) << 16);

@@ -320,6 +320,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.tokens_per_module = D.N;
   g.usum = ra.usum;
   g.sy = ra.sy;
+  g.aux_slots = L.aux_slots;
   plan_units(g, sms, false);
   if (!mark(SOLO_STAGE_LOGITS) ||
       fail(launch_gemm(affine ? kLogitsHeads : kLogits, mX_k, mW_k, mP_st, mAux, g, sms,
@@ -660,6 +661,8 @@ const char* solo_readout_strerror(solo_status_t status) {
 int32_t solo_readout_version(void) { return 100; }
 
 uint64_t solo_readout_kernel_launches(void) { return solo::launch_count(); }
+
+int32_t solo_readout_build_flags(void) { return SOLO_DEBUG ? SOLO_BUILD_CHECKED : 0; }
 
 }  // extern "C"
 

@@ -54,7 +54,9 @@ _lib = None
 
 
 def library_path() -> str:
-    return _build.LIB
+    """The in-tree release library, or the file named by SOLO_READOUT_LIB (e.g.
+    the checked build)."""
+    return os.environ.get("SOLO_READOUT_LIB") or _build.LIB
 
 
 def load(path: str | None = None) -> ctypes.CDLL:
@@ -111,6 +113,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_version.restype = i32
     lib.solo_readout_kernel_launches.argtypes = []
     lib.solo_readout_kernel_launches.restype = ctypes.c_uint64
+    lib.solo_readout_build_flags.argtypes = []
+    lib.solo_readout_build_flags.restype = i32
     _lib = lib
     return lib
 
@@ -350,6 +354,11 @@ def solo_readout_selftest_wait_timeout(device_flags, limit_us: int, stream=None,
 
 def solo_readout_version() -> int:
     return load().solo_readout_version()
+
+
+def solo_readout_build_flags() -> int:
+    """SOLO_BUILD_CHECKED (1) when the loaded library is the checked build."""
+    return int(load().solo_readout_build_flags())
 
 
 def solo_readout_kernel_launches() -> int:

@@ -173,3 +173,14 @@ def test_launch_counter_ignores_rejected_calls(sr):
                                    a["workspace"], workspace_bytes=1024, stream=0,
                                    check=False) == sr.SOLO_ERR_WORKSPACE_TOO_SMALL
     assert sr.solo_readout_kernel_launches() == before
+
+
+def test_checked_build_exports_and_reports_itself(built_library):
+    """The bounds-checked twin exports every declared symbol and says which it is."""
+    from paper_2609_35440_gb300 import build as b
+    path = b.LIB_CHECKED if b.up_to_date_checked() else b.build(checked=True)
+    chk = ctypes.CDLL(path)
+    for name in declared_functions():
+        assert hasattr(chk, name), name
+    assert chk.solo_readout_build_flags() == 1
+    assert ctypes.CDLL(built_library).solo_readout_build_flags() == 0
