@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   for (int j = 0; j < 8; ++j) colsum[j] = 0.f;
   uint4* P = reinterpret_cast<uint4*>(a.P + row0 * a.ldp) + vec;
   const int64_t stride = a.ldp / 8;
-  constexpr int kAhead = 4;                           // rows in flight per thread
+  constexpr int kAhead = 8;                           // rows in flight per thread
   for (int r0 = 0; r0 < rows; r0 += kAhead) {
     uint4 in[kAhead];
 #pragma unroll
