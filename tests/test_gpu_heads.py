@@ -70,6 +70,33 @@ def test_heads_small_full_parity(sr, wl):
     print(wl.name, rep)
 
 
+@pytest.mark.parametrize("neg_tau,bias_std", [(True, 0.5), (False, 25.0)],
+                         ids=["negative_tau", "wide_bias"])
+def test_heads_reference_choices(sr, neg_tau, bias_std):
+    """Temperatures of both signs (the first pass bounds tau s from the other
+    side), and biases spanning far more than 60 within a tile (the first pass
+    falls back to forming every z), both against the oracle."""
+    wl = Workload("heads_k3_n200_d136_v1001", K=3, N=200, d=136, V=1001, seed=64,
+                  mask_frac=0.05)
+    inp = synth.generate(wl)
+    tau, bias = synth.gen_heads(wl, bias_std=bias_std)
+    if neg_tau:
+        tau[0] = -0.7
+    else:   # the tiles' bias spans exceed 60
+        assert np.min(np.ptp(bias[:, :256], axis=1)) > 60.0
+    gpu = _gpu(sr, wl, inp, tau, bias)
+    assert gpu["flags"] == 0
+    dec = orc.bf16_bits_to_f64
+    ref = orc.solo_readout_fwd_bwd([dec(inp.hidden[k]) for k in range(wl.K)], dec(inp.gamma),
+                                   dec(inp.W), inp.targets.astype(np.int64),
+                                   eps=float(np.float32(wl.eps)), tau=tau.astype(np.float64),
+                                   bias=bias.astype(np.float64))
+    rep = parity.compare_full(wl, gpu, ref)
+    parity.check_grad("dtau", gpu["dtau"], ref["dtau"], rep)
+    for k in range(wl.K):
+        parity.check_grad(f"dbias[{k}]", gpu["dbias"][k], ref["dbias"][k], rep)
+
+
 def test_without_heads_is_the_plain_call_bitwise(sr):
     wl = SMALL[1]
     inp = synth.generate(wl)
