@@ -18,8 +18,9 @@ steps, a barrier and a device synchronize on both sides of the timed region.
 ``e2e`` repeats the measurement through the same C ABI call with every step's
 inputs copied from pinned host memory (on a copy stream, into one of two
 device buffers, overlapping the previous step's compute) and its losses read
-back, all inside the timed region.  ``cpu_baseline`` times the fp64 oracle on a bounded sample
-of the same workload on the host cores.
+back, all inside the timed region.  ``cpu_baseline`` times the fp64 oracle
+on a bounded sample of the same workload on the host cores.  ``gpu_launches``
+is the library's own count of the kernels it enqueued during the timed calls.
 """
 from __future__ import annotations
 
