@@ -120,3 +120,37 @@ def test_exit_readout_full_size_sampled(sr, wl):
         want = gpu["loss_tok"][k][kept].sum() / kept.sum()
         assert abs(gpu["loss_mean"][k] - want) <= 1e-6 * want
     print(wl.name, rep)
+
+
+def test_exit_top1_ties_take_the_first_index(sr):
+    """Readout rows copied to later positions (within a 32-column chunk, across
+    chunks of a tile and across 256-column tiles) give exactly equal logits on
+    the GPU; the top-1 is then the lowest index among the tied copies (the first
+    maximum).  The oracle's logits are made exactly tied the same way (a copy
+    takes its source's value) before its first argmax is taken."""
+    wl = Workload("ties_k2_n256_d128_v1001", K=2, N=256, d=128, V=1001, seed=52)
+    inp = synth.generate(wl)
+    W = inp.W.copy()
+    root = np.arange(wl.V)
+    for dst, src in ((np.arange(1, 256, 2), np.arange(0, 256, 2)),     # same chunk
+                     (np.arange(256, 512), np.arange(0, 256)),         # next tile
+                     (np.arange(700, 740), np.arange(600, 640))):      # other chunks, tiles
+        W[dst] = W[src]
+        root[dst] = root[src]
+    inp.W = W
+    gpu = _gpu_exit(sr, wl, inp, with_targets=False)
+    assert gpu["flags"] == 0
+    dec = orc.bf16_bits_to_f64
+    ties_seen = 0
+    for k in range(wl.K):
+        ref = orc.exit_readout([dec(inp.hidden[k])], dec(inp.gamma), dec(W), None, None,
+                               eps=float(np.float32(wl.eps)), contract=True)
+        z = ref["z"][0][:, root]                  # copies take exactly their source's value
+        want = np.argmax(z, axis=1)               # first maximum
+        best_root = root[want]
+        other = np.where(root[None, :] == best_root[:, None], -np.inf, z)
+        zmax = z[np.arange(wl.N), want]
+        clear = zmax - other.max(axis=1) > 1e-3 * np.maximum(1.0, np.abs(zmax))
+        assert np.array_equal(gpu["top1"][k][clear], want[clear])
+        ties_seen += int(np.sum(clear & (np.sum(z == zmax[:, None], axis=1) > 1)))
+    assert ties_seen > 0

@@ -155,3 +155,36 @@ def test_kernel_launch_counter():
     assert 10 <= full <= 12
     # without dW and dgamma: no dW GEMM (nor its fix-up), dgamma parts or reduction
     assert 7 <= count(want_dW=False, want_dgamma=False) <= full - 3
+
+
+def test_zero_readout_closed_forms():
+    """W = 0: every logit is 0, so each kept token's loss is ln V, dH and dgamma
+    are exactly zero, and dW = (1/Nvalid) sum_i (1/V - e_{y_i}) xhat_i^T for the
+    final module (the closed form, evaluated in fp64 from the GPU's own inputs)."""
+    import oracle.solo_oracle as orc
+    wl = Workload("zeroW_k2_n300_d136_v1001", K=2, N=300, d=136, V=1001, seed=47,
+                  mask_frac=0.1)
+    inp = synth.generate(wl)
+    inp.W = np.zeros_like(inp.W)
+    gpu = parity.run_gpu(wl, inp)
+    assert gpu["flags"] == 0
+    kept = inp.targets != wl.ignore_index
+    lnV = np.log(wl.V)
+    assert np.max(np.abs(gpu["loss_tok"][kept] - lnV)) <= 1e-5
+    assert np.all(gpu["loss_tok"][~kept] == 0.0)
+    assert np.allclose(gpu["loss_mean"], lnV, rtol=1e-6, atol=0.0)
+    for k in range(wl.K):
+        assert not np.any(gpu["dhidden"][k])
+    assert not np.any(gpu["dgamma"])
+    # dW of the final module from its x-hat (rounded exactly as the GPU rounds it)
+    dec = orc.bf16_bits_to_f64
+    k = wl.K - 1
+    xhat = orc.rmsnorm_forward(dec(inp.hidden[k]), dec(inp.gamma), float(np.float32(wl.eps)),
+                               contract=True)[1]
+    y = inp.targets[k]
+    keep = y != wl.ignore_index
+    g = np.zeros((wl.N, wl.V))
+    g[keep] = 1.0 / wl.V
+    g[np.flatnonzero(keep), y[keep]] -= 1.0
+    want = g.T @ xhat / keep.sum()
+    parity.check_grad("dW (W = 0)", gpu["dW"], want, {})
