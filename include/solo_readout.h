@@ -304,6 +304,25 @@ solo_status_t solo_readout_fwd_bwd_private(const solo_dims_t* dims,
                                            solo_stream_t stream);
 
 /*
+ * The final RMSNorm alone (the first step of every call): for each module k
+ * and token i, r_i = (mean_j h_ij^2 + eps)^-1/2 and xhat_ij = bf16(gamma_j
+ * h_ij r_i), rounded to nearest even on the exact value of gamma h r (paper,
+ * Section 2.2: the head's final RMSNorm with element-wise gain), i.e. the
+ * x-hat that the readout multiplies.  Of dims, K, N, d and eps are used (V
+ * must still be valid).
+ *
+ *  hidden  host array [K] of device pointers, each bf16 [N, d].
+ *  gamma   bf16 [d].
+ *  xhat    bf16 [K*N, d], module-major rows: row k*N + i is token i of module k.
+ *  r       fp32 [K*N] or NULL.
+ *
+ * Asynchronous on `stream`; allocates nothing.
+ */
+solo_status_t solo_readout_rmsnorm(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                                   const solo_bf16_t* gamma, solo_bf16_t* xhat, float* r,
+                                   solo_stream_t stream);
+
+/*
  * Waits for `stream`, then copies the flag word of the last call that used
  * `workspace` into *flags (host).  The word is cleared at the start of
  * every call.

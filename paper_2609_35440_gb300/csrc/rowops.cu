@@ -185,7 +185,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   } else {
     for (int v = lane; v < nv; v += 32) emit(v, __ldg(h + v));
   }
-  if (lane == 0) a.r[row] = r;
+  if (lane == 0 && a.r) a.r[row] = r;
 }
 
 // ---- log-sum-exp over column tiles, token loss, per-block module sums ----------

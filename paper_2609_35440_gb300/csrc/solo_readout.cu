@@ -630,6 +630,38 @@ solo_status_t solo_readout_fwd_bwd_private(
   return SOLO_OK;
 }
 
+solo_status_t solo_readout_rmsnorm(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                                   const solo_bf16_t* gamma, solo_bf16_t* xhat, float* r,
+                                   solo_stream_t stream) {
+  solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  const solo_dims_t& D = *dims;
+  if (hidden == nullptr || gamma == nullptr || xhat == nullptr) return SOLO_ERR_INVALID_ARG;
+  for (int k = 0; k < D.K; ++k) {
+    if (hidden[k] == nullptr) return SOLO_ERR_INVALID_ARG;
+    if (!aligned16(hidden[k])) return SOLO_ERR_MISALIGNED;
+  }
+  if (!aligned16(gamma) || !aligned16(xhat) || (reinterpret_cast<uintptr_t>(r) & 3u))
+    return SOLO_ERR_MISALIGNED;
+  int sms = 0;
+  st = device_setup(&sms);
+  if (st != SOLO_OK) return st;
+  RowArgs ra;
+  std::memset(&ra, 0, sizeof(ra));
+  for (int k = 0; k < D.K; ++k) ra.hidden[k] = hidden[k];
+  ra.N = D.N;
+  ra.K = D.K;
+  ra.d = D.d;
+  ra.V = D.V;
+  ra.eps = D.eps;
+  ra.gamma = gamma;
+  ra.xhat = xhat;
+  ra.r = r;
+  return launch_rmsnorm_fwd(ra, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? SOLO_OK
+             : SOLO_ERR_CUDA;
+}
+
 solo_status_t solo_readout_get_flags(const void* workspace, solo_stream_t stream,
                                      uint32_t* flags) {
   if (workspace == nullptr || flags == nullptr) return SOLO_ERR_INVALID_ARG;

@@ -115,6 +115,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_kernel_launches.restype = ctypes.c_uint64
     lib.solo_readout_build_flags.argtypes = []
     lib.solo_readout_build_flags.restype = i32
+    lib.solo_readout_rmsnorm.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp]
+    lib.solo_readout_rmsnorm.restype = i32
     _lib = lib
     return lib
 
@@ -354,6 +356,19 @@ def solo_readout_selftest_wait_timeout(device_flags, limit_us: int, stream=None,
 
 def solo_readout_version() -> int:
     return load().solo_readout_version()
+
+
+def solo_readout_rmsnorm(dims: solo_dims_t, hidden: Sequence, gamma, xhat, r=None, stream=None,
+                         check: bool = True) -> int:
+    """The final RMSNorm alone: xhat bf16 [K*N, d] and, optionally, r fp32 [K*N]."""
+    if len(hidden) != dims.K:
+        raise ValueError("hidden needs K entries")
+    harr = (ctypes.c_void_p * dims.K)(*[_ptr(h) for h in hidden])
+    st = load().solo_readout_rmsnorm(ctypes.byref(dims), harr, _ptr(gamma), _ptr(xhat), _ptr(r),
+                                     _stream_handle(stream))
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_rmsnorm")
+    return st
 
 
 def solo_readout_build_flags() -> int:

@@ -184,3 +184,16 @@ def test_checked_build_exports_and_reports_itself(built_library):
         assert hasattr(chk, name), name
     assert chk.solo_readout_build_flags() == 1
     assert ctypes.CDLL(built_library).solo_readout_build_flags() == 0
+
+
+def test_rmsnorm_host_checks(sr):
+    fake = 1 << 20
+    dims = sr.make_dims(2, 16, 64, 100)
+    assert sr.solo_readout_rmsnorm(dims, [fake, None], fake, fake, stream=0,
+                                   check=False) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_rmsnorm(dims, [fake, fake], fake, None, stream=0,
+                                   check=False) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_rmsnorm(dims, [fake, fake], fake, fake + 8, stream=0,
+                                   check=False) == sr.SOLO_ERR_MISALIGNED
+    assert sr.solo_readout_rmsnorm(sr.make_dims(2, 16, 60, 100), [fake, fake], fake, fake,
+                                   stream=0, check=False) == sr.SOLO_ERR_UNSUPPORTED_SHAPE
