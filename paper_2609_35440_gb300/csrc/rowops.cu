@@ -104,6 +104,25 @@ __device__ __forceinline__ uint16_t xhat_bf16(float gh, F2 r) {
   return static_cast<uint16_t>((b + 0x7FFFu + ((b >> 16) & 1u)) >> 16);
 }
 
+// True when fp32 y lies within 4 ulp of a bf16 midpoint (|low 16 bits - 0x8000| <= 4).
+__device__ __forceinline__ bool near_midpoint(float y) {
+  return ((__float_as_uint(y) - 0x7FFCu) & 0xFFFFu) <= 8u;
+}
+
+// Two x-hat values: away from midpoints the fp32 product rounds like the exact
+// value, and the hardware's round-to-nearest-even packs both; otherwise each
+// takes the exact test of xhat_bf16.
+__device__ __forceinline__ uint32_t xhat_bf16x2(float gh0, float gh1, F2 r) {
+  const float y0 = gh0 * r.hi;
+  const float y1 = gh1 * r.hi;
+  if (near_midpoint(y0) || near_midpoint(y1))
+    return static_cast<uint32_t>(xhat_bf16(gh0, r)) |
+           (static_cast<uint32_t>(xhat_bf16(gh1, r)) << 16);
+  uint32_t w;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w) : "f"(y1), "f"(y0));
+  return w;
+}
+
 // VPL > 0: the row is held in registers (VPL 16-byte vectors per lane, d <=
 // 256 * VPL), so h is read from memory once.  VPL == 0: any d, h re-read.
 template <int VPL>
@@ -169,11 +188,8 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
     unpack8(__ldg(g + v), gg);
     uint32_t w[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t lo = xhat_bf16(gg[2 * j] * f[2 * j], rr);
-      const uint32_t hi = xhat_bf16(gg[2 * j + 1] * f[2 * j + 1], rr);
-      w[j] = lo | (hi << 16);
-    }
+    for (int j = 0; j < 4; ++j)
+      w[j] = xhat_bf16x2(gg[2 * j] * f[2 * j], gg[2 * j + 1] * f[2 * j + 1], rr);
     out[v] = make_uint4(w[0], w[1], w[2], w[3]);
   };
   if constexpr (VPL > 0) {
