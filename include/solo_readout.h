@@ -128,7 +128,9 @@ solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* byte
  *  workspace  device buffer of at least solo_readout_workspace_bytes bytes,
  *             16-byte aligned; its contents on entry do not matter.
  *
- * Output buffers may not alias inputs or each other.  Returns SOLO_OK once
+ * Output buffers (and the workspace) may not overlap inputs or each other;
+ * an overlap is refused with SOLO_ERR_INVALID_ARG before anything is
+ * enqueued (inputs may share memory).  Returns SOLO_OK once
  * the work is enqueued.
  */
 solo_status_t solo_readout_fwd_bwd(const solo_dims_t* dims,

@@ -117,6 +117,30 @@ Layout make_layout(const solo_dims_t& d) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Byte ranges of a call's buffers: an output (or the workspace) may overlap
+// no other buffer; inputs may share memory with each other (they are only
+// read).
+struct Ranges {
+  static constexpr int kMax = 2 * SOLO_MAX_MODULES + 16;
+  uintptr_t lo[kMax];
+  uintptr_t hi[kMax];
+  bool out[kMax];
+  int n = 0;
+  void add(const void* p, size_t bytes, bool is_out) {
+    if (p == nullptr || bytes == 0 || n == kMax) return;
+    lo[n] = reinterpret_cast<uintptr_t>(p);
+    hi[n] = lo[n] + bytes;
+    out[n] = is_out;
+    ++n;
+  }
+  bool any_output_overlap() const {
+    for (int i = 0; i < n; ++i)
+      for (int j = i + 1; j < n; ++j)
+        if ((out[i] || out[j]) && lo[i] < hi[j] && lo[j] < hi[i]) return true;
+    return false;
+  }
+};
+
 // ---- per-device setup ------------------------------------------------------------
 
 struct DeviceInfo {
@@ -216,6 +240,29 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   const bool affine = tau || bias || dtau;   // z = tau s + b (and its temperature gradient)
   const Layout L = make_layout(D);
   if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+  {
+    const size_t K = static_cast<size_t>(D.K), N = static_cast<size_t>(D.N);
+    const size_t dd = static_cast<size_t>(D.d), VV = static_cast<size_t>(D.V);
+    Ranges rg;
+    for (int k = 0; k < D.K; ++k) {
+      rg.add(hidden[k], N * dd * 2, false);
+      rg.add(dhidden[k], N * dd * 2, true);
+    }
+    rg.add(gamma, dd * 2, false);
+    rg.add(W, VV * dd * 2, false);
+    rg.add(targets, K * N * 4, false);
+    rg.add(mask, K * N, false);
+    rg.add(tau, K * 4, false);
+    rg.add(bias, K * VV * 4, false);
+    rg.add(loss_tok, K * N * 4, true);
+    rg.add(loss_mean, K * 4, true);
+    rg.add(dW, VV * dd * 4, true);
+    rg.add(dgamma, dd * 4, true);
+    rg.add(dtau, K * 4, true);
+    rg.add(dbias, K * VV * 4, true);
+    rg.add(workspace, L.total, true);
+    if (rg.any_output_overlap()) return SOLO_ERR_INVALID_ARG;
+  }
 
   // -------- device
   int sms = 0;

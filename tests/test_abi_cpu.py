@@ -197,3 +197,28 @@ def test_rmsnorm_host_checks(sr):
                                    check=False) == sr.SOLO_ERR_MISALIGNED
     assert sr.solo_readout_rmsnorm(sr.make_dims(2, 16, 60, 100), [fake, fake], fake, fake,
                                    stream=0, check=False) == sr.SOLO_ERR_UNSUPPORTED_SHAPE
+
+
+def test_overlapping_outputs_are_refused(sr):
+    """An output that overlaps an input, another output or the workspace is
+    refused before any launch; inputs may share memory."""
+    base = 1 << 30
+    K, N, d, V = 2, 16, 64, 100
+    mb = 1 << 20
+    ptr = {name: base + i * mb for i, name in enumerate(
+        ["h0", "h1", "g", "W", "t", "lm", "dh0", "dh1", "dW", "dg", "lt", "ws"])}
+
+    def call(**over):
+        p = dict(ptr, **over)
+        return sr.solo_readout_fwd_bwd(sr.make_dims(K, N, d, V), [p["h0"], p["h1"]], p["g"],
+                                       p["W"], p["t"], None, p["lt"], p["lm"],
+                                       [p["dh0"], p["dh1"]], p["dW"], p["dg"], p["ws"],
+                                       workspace_bytes=1 << 40, stream=0, check=False)
+
+    assert call(dW=ptr["W"]) == sr.SOLO_ERR_INVALID_ARG                 # output on an input
+    assert call(dh0=ptr["h1"] + 256) == sr.SOLO_ERR_INVALID_ARG         # partial overlap
+    assert call(dh1=ptr["dh0"]) == sr.SOLO_ERR_INVALID_ARG              # two outputs
+    assert call(lm=ptr["ws"] + 4096) == sr.SOLO_ERR_INVALID_ARG         # inside the workspace
+    # inputs sharing memory pass this check (the call then needs a GPU)
+    assert call(h1=ptr["h0"]) != sr.SOLO_ERR_INVALID_ARG
+    assert call() != sr.SOLO_ERR_INVALID_ARG
