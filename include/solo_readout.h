@@ -190,6 +190,8 @@ solo_status_t solo_readout_fwd_bwd_events(const solo_dims_t* dims,
  * Runs the RMSNorm, one tensor-core pass over the vocabulary (K*2NVd FLOPs)
  * and a combine; no exponential or gradient buffer is written.  Flags as for
  * solo_readout_fwd_bwd (read with solo_readout_get_flags on this workspace).
+ * Outputs and the workspace may not overlap inputs or each other
+ * (SOLO_ERR_INVALID_ARG).
  */
 solo_status_t solo_readout_exit_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
 solo_status_t solo_readout_exit_forward(const solo_dims_t* dims,
@@ -318,7 +320,8 @@ solo_status_t solo_readout_fwd_bwd_private(const solo_dims_t* dims,
  *  xhat    bf16 [K*N, d], module-major rows: row k*N + i is token i of module k.
  *  r       fp32 [K*N] or NULL.
  *
- * Asynchronous on `stream`; allocates nothing.
+ * Asynchronous on `stream`; allocates nothing.  xhat and r may not overlap
+ * the inputs or each other (SOLO_ERR_INVALID_ARG).
  */
 solo_status_t solo_readout_rmsnorm(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
                                    const solo_bf16_t* gamma, solo_bf16_t* xhat, float* r,

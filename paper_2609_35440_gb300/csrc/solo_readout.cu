@@ -473,6 +473,21 @@ solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden
     return SOLO_ERR_MISALIGNED;
   const ExitLayout L = make_exit_layout(D);
   if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+  {
+    const size_t K = static_cast<size_t>(D.K), N = static_cast<size_t>(D.N);
+    Ranges rg;
+    for (int k = 0; k < D.K; ++k) rg.add(hidden[k], N * D.d * 2, false);
+    rg.add(gamma, static_cast<size_t>(D.d) * 2, false);
+    rg.add(W, static_cast<size_t>(D.V) * D.d * 2, false);
+    rg.add(targets, K * N * 4, false);
+    rg.add(mask, K * N, false);
+    rg.add(loss_tok, K * N * 4, true);
+    rg.add(loss_mean, K * 4, true);
+    rg.add(top1, K * N * 4, true);
+    rg.add(top1_logprob, K * N * 4, true);
+    rg.add(workspace, L.total, true);
+    if (rg.any_output_overlap()) return SOLO_ERR_INVALID_ARG;
+  }
   int sms = 0;
   st = device_setup(&sms);
   if (st != SOLO_OK) return st;
@@ -690,6 +705,15 @@ solo_status_t solo_readout_rmsnorm(const solo_dims_t* dims, const solo_bf16_t* c
   }
   if (!aligned16(gamma) || !aligned16(xhat) || (reinterpret_cast<uintptr_t>(r) & 3u))
     return SOLO_ERR_MISALIGNED;
+  {
+    const size_t M = static_cast<size_t>(D.K) * D.N;
+    Ranges rg;
+    for (int k = 0; k < D.K; ++k) rg.add(hidden[k], static_cast<size_t>(D.N) * D.d * 2, false);
+    rg.add(gamma, static_cast<size_t>(D.d) * 2, false);
+    rg.add(xhat, M * D.d * 2, true);
+    rg.add(r, M * 4, true);
+    if (rg.any_output_overlap()) return SOLO_ERR_INVALID_ARG;
+  }
   int sms = 0;
   st = device_setup(&sms);
   if (st != SOLO_OK) return st;

@@ -222,3 +222,19 @@ def test_overlapping_outputs_are_refused(sr):
     # inputs sharing memory pass this check (the call then needs a GPU)
     assert call(h1=ptr["h0"]) != sr.SOLO_ERR_INVALID_ARG
     assert call() != sr.SOLO_ERR_INVALID_ARG
+
+
+def test_exit_and_rmsnorm_overlaps_are_refused(sr):
+    base, mb = 1 << 30, 1 << 20
+    dims = sr.make_dims(2, 16, 64, 100)
+    h0, h1, g, W, t, lt, lm, top, tlp, ws = (base + i * mb for i in range(10))
+    exit_call = lambda **o: sr.solo_readout_exit_forward(
+        dims, [h0, h1], g, W, t, None, o.get("lt", lt), lm, o.get("top", top), tlp, ws,
+        workspace_bytes=1 << 40, stream=0, check=False)
+    assert exit_call(top=W) == sr.SOLO_ERR_INVALID_ARG
+    assert exit_call(lt=top) == sr.SOLO_ERR_INVALID_ARG
+    assert exit_call() != sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_rmsnorm(dims, [h0, h1], g, h1, stream=0,
+                                   check=False) == sr.SOLO_ERR_INVALID_ARG
+    assert sr.solo_readout_rmsnorm(dims, [h0, h1], g, W, stream=0,
+                                   check=False) != sr.SOLO_ERR_INVALID_ARG
