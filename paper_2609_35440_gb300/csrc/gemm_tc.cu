@@ -53,8 +53,9 @@ namespace {
 
 constexpr int kPairRows = 2 * kBM;                  // 256 output rows per CTA pair
 constexpr int kBHalf = kBN / 2;                     // B columns staged per CTA
-constexpr int kABytes = kBM * kBK * 2;              // 16 KB
-constexpr int kBBytes = kBHalf * kBK * 2;           // 16 KB
+constexpr int kABytes = kBM * kBK * 2;              // 16 KB at kBK = 64
+constexpr int kBBytes = kBHalf * kBK * 2;           // 16 KB at kBK = 64
+constexpr int kMnBlock = 64 * kBK * 2;              // MN-major: one 64-wide MN block
 constexpr int kStageBytes = kABytes + kBBytes;      // per CTA
 constexpr int kEpiBufBytes = 32 * 128;              // 32 rows x 128 B
 constexpr int kEpiWarps = 4;
@@ -193,18 +194,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           const uint32_t fb = full_even + stage * 8;
           const int kr = args.k_row0 + kb * kBK;
           if constexpr (!kAmn) {
-            tma_load_2d_pair(sA, &tmA, fb, kb * kBK, m0);
+#pragma unroll
+            for (int a = 0; a < kKAtoms; ++a)
+              tma_load_2d_pair(sA + a * kBM * 128, &tmA, fb, kb * kBK + 64 * a, m0);
           } else {
 #pragma unroll
             for (int c = 0; c < kBM / 64; ++c)
-              tma_load_2d_pair(sA + c * 8192, &tmA, fb, m0 + 64 * c, kr);
+              tma_load_2d_pair(sA + c * kMnBlock, &tmA, fb, m0 + 64 * c, kr);
           }
           if constexpr (!kBmn) {
-            tma_load_2d_pair(sB, &tmB, fb, kb * kBK, n0);
+#pragma unroll
+            for (int a = 0; a < kKAtoms; ++a)
+              tma_load_2d_pair(sB + a * kBHalf * 128, &tmB, fb, kb * kBK + 64 * a, n0);
           } else {
 #pragma unroll
             for (int c = 0; c < kBHalf / 64; ++c)
-              tma_load_2d_pair(sB + c * 8192, &tmB, fb, n0 + 64 * c, kr);
+              tma_load_2d_pair(sB + c * kMnBlock, &tmB, fb, n0 + 64 * c, kr);
           }
           issued |= 1u << stage;
           last_phase = (last_phase & ~(1u << stage)) | (phase << stage);
@@ -266,10 +271,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           const uint32_t sb = b_base + stage * kBBytes;
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
-            const uint64_t ad = kAmn ? smem_desc_sw128(sa + k * 2048, 8192, 1024)
-                                     : smem_desc_sw128(sa + k * 32, 16, 1024);
-            const uint64_t bd = kBmn ? smem_desc_sw128(sb + k * 2048, 8192, 1024)
-                                     : smem_desc_sw128(sb + k * 32, 16, 1024);
+            // K-major: 16-wide K steps within a 64-wide swizzle atom, atoms one
+            // after the other; MN-major: 16 K rows of 128 B, MN blocks kMnBlock apart
+            const uint64_t ad =
+                kAmn ? smem_desc_sw128(sa + k * 2048, kMnBlock, 1024)
+                     : smem_desc_sw128(sa + (k / 4) * kBM * 128 + (k % 4) * 32, 16, 1024);
+            const uint64_t bd =
+                kBmn ? smem_desc_sw128(sb + k * 2048, kMnBlock, 1024)
+                     : smem_desc_sw128(sb + (k / 4) * kBHalf * 128 + (k % 4) * 32, 16, 1024);
             mma_bf16_pair(d_tmem, ad, bd, kIdesc, (kb != kb_lo || k != 0) ? 1u : 0u);
           }
           mma_commit_pair(&empty[stage], kBothCtas);

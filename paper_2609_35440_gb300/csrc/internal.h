@@ -40,8 +40,13 @@ inline cudaError_t launched() {
 // 128 rows), reduction in blocks of 64 through a 6-stage shared-memory ring.
 constexpr int kBM = 128;
 constexpr int kBN = 256;
-constexpr int kBK = 64;
-constexpr int kStages = 6;
+#ifndef SOLO_GEMM_BK
+#define SOLO_GEMM_BK 128
+#endif
+constexpr int kBK = SOLO_GEMM_BK;          // 64 or 128 bf16 elements per reduction block
+static_assert(kBK == 64 || kBK == 128, "reduction block");
+constexpr int kStages = 6 * 64 / kBK;      // 192 KB of operand ring per CTA
+constexpr int kKAtoms = kBK / 64;          // 128-byte swizzle atoms along K per row
 constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
 // The three products of one call.

@@ -321,13 +321,13 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
   CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW, mAux;
   float* aux = reinterpret_cast<float*>(ws + L.aux);
-  bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, kBK, kBM) &&
+  bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, 64, kBM) &&
             make_map(&mAux, F32, aux, kBN,
                      static_cast<uint64_t>(std::max(L.aux_slots, 1)) * 2 * kBM, kBN * 4, 32,
                      32) &&
-            make_map(&mW_k, BF, W, d, V, d * 2, kBK, kBN / 2) &&
+            make_map(&mW_k, BF, W, d, V, d * 2, 64, kBN / 2) &&
             make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
-            make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, kBK, kBM) &&
+            make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBM) &&
             make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK) &&
             make_map(&mDX, F32, ra.dxhat, d, M, d * 4, 32, 32);
   if (ok && dW) {
@@ -525,8 +525,8 @@ solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden
   const uint64_t d = static_cast<uint64_t>(D.d);
   const uint64_t V = static_cast<uint64_t>(D.V);
   CUtensorMap mX_k, mW_k;
-  if (!make_map(&mX_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ra.xhat, d, M, d * 2, kBK, kBM) ||
-      !make_map(&mW_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, W, d, V, d * 2, kBK, kBN / 2))
+  if (!make_map(&mX_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ra.xhat, d, M, d * 2, 64, kBM) ||
+      !make_map(&mW_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, W, d, V, d * 2, 64, kBN / 2))
     return SOLO_ERR_CUDA;
   auto mark = [&](int stage) -> bool {
     if (events == nullptr) return true;
