@@ -3,10 +3,10 @@
 // Two CTAs on neighbouring SMs form a cluster and compute one 256 x 256
 // output tile together with tcgen05.mma.cta_group::2 (M = 256, N = 256, K =
 // 16, bf16 in, fp32 accumulate).  Each CTA stages its own 128 rows of A and
-// its own 128 columns of B per 64-wide reduction block (32 KB), so a 6-stage
-// ring fits in shared memory and each SM needs 64 B of operands per clock at
-// full MMA rate (a single-CTA 128 x 256 tile needs 96 B and only has room
-// for 4 stages).  Roles, in both CTAs:
+// its own 128 columns of B per 128-wide reduction block (64 KB), so a
+// 3-stage ring fits in shared memory next to the epilogue's staging buffers,
+// and each SM needs 64 B of operands per clock at full MMA rate (a single-CTA
+// 128 x 256 tile needs 96 B).  Roles, in both CTAs:
 //   warp 0     TMA producer: loads its CTA's A and B halves, completion is
 //              signalled on the even CTA's "full" barrier (pair-mode TMA)
 //   warp 1     even CTA: one thread issues the pair MMAs into one of two TMEM
@@ -54,8 +54,8 @@ namespace {
 
 constexpr int kPairRows = 2 * kBM;                  // 256 output rows per CTA pair
 constexpr int kBHalf = kBN / 2;                     // B columns staged per CTA
-constexpr int kABytes = kBM * kBK * 2;              // 16 KB at kBK = 64
-constexpr int kBBytes = kBHalf * kBK * 2;           // 16 KB at kBK = 64
+constexpr int kABytes = kBM * kBK * 2;              // 32 KB at kBK = 128
+constexpr int kBBytes = kBHalf * kBK * 2;           // 32 KB at kBK = 128
 constexpr int kMnBlock = 64 * kBK * 2;              // MN-major: one 64-wide MN block
 constexpr int kStageBytes = kABytes + kBBytes;      // per CTA
 constexpr int kEpiBufBytes = 32 * 128;              // 32 rows x 128 B

@@ -37,7 +37,7 @@ inline cudaError_t launched() {
 }
 
 // Tensor-core tile: a CTA pair computes 256 rows x 256 columns (each CTA owns
-// 128 rows), reduction in blocks of 64 through a 6-stage shared-memory ring.
+// 128 rows), reduction in blocks of kBK through a shared-memory ring.
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 #ifndef SOLO_GEMM_BK
@@ -49,7 +49,7 @@ constexpr int kStages = 6 * 64 / kBK;      // 192 KB of operand ring per CTA
 constexpr int kKAtoms = kBK / 64;          // 128-byte swizzle atoms along K per row
 constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
-// The three products of one call.
+// The products of the GEMM kernel.
 enum GemmMode : int {
   kLogits = 0,  // Z = Xhat W^T (A: Xhat K-major, B: W K-major); epilogue: per-tile
                 //   max / sum of exp, target logit, bf16 exp(z - tile max) stored
