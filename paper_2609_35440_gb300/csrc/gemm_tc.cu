@@ -415,20 +415,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         float mx = -INFINITY, zyv = 0.f, syv = 0.f;
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
-          float v[32], bb[32];
+          float v[32], bb[32], z[32];
           tmem_ld32(tbase + c * 32, v);
           if constexpr (kHeads) load_bias(c, bb);
-          const int yc = has_y ? yrel - c * 32 : -1;   // target column within this chunk
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float z = kHeads ? fmaf(tau, v[j], bb[j]) : v[j];
-            if (c * 32 + j < ncols) mx = fmaxf(mx, z);
-            zyv = (j == yc) ? z : zyv;
-            if constexpr (kHeads) syv = (j == yc) ? v[j] : syv;
+          for (int j = 0; j < 32; ++j) z[j] = kHeads ? fmaf(tau, v[j], bb[j]) : v[j];
+          // the target logit, in the chunks holding some lane's target only
+          const int yc = has_y ? yrel - c * 32 : -1;
+          if (__any_sync(0xffffffffu, static_cast<unsigned>(yc) < 32u)) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              zyv = (j == yc) ? z[j] : zyv;
+              if constexpr (kHeads) syv = (j == yc) ? v[j] : syv;
+            }
           }
+          if (c * 32 + 32 > ncols) {              // ragged last chunk (warp-uniform)
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (c * 32 + j >= ncols) z[j] = -INFINITY;
+          }
+          // max of mx and the 32 values: a tree of three-input maxima
+          float t[11];
+#pragma unroll
+          for (int i = 0; i < 10; ++i) t[i] = fmax3(z[3 * i], z[3 * i + 1], z[3 * i + 2]);
+          t[10] = fmax3(z[30], z[31], mx);
+          mx = fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]),
+                     fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
         }
         const float mlog = mx * kLog2e;
-        float ssum = 0.f, usum = 0.f;
+        // the sum of exp(z - m) in two lanes of a packed pair (even and odd columns)
+        float2 sacc = make_float2(0.f, 0.f);
+        float usum = 0.f;
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
           if (lane == 0) bulk_wait_group_read<1>();
@@ -446,14 +463,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               for (int j = 0; j < 32; ++j) v[j] = bb[j] = 0.f;
             }
             uint32_t p[16];
+            const bool ragged = c * 32 + 32 > ncols;      // warp-uniform
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              const int col = c * 32 + 2 * j;
-              const float z0 = kHeads ? fmaf(tau, v[2 * j], bb[2 * j]) : v[2 * j];
-              const float z1 = kHeads ? fmaf(tau, v[2 * j + 1], bb[2 * j + 1]) : v[2 * j + 1];
-              const float e0 = col < ncols ? ex2_approx(fmaf(z0, kLog2e, -mlog)) : 0.f;
-              const float e1 = col + 1 < ncols ? ex2_approx(fmaf(z1, kLog2e, -mlog)) : 0.f;
-              ssum += e0 + e1;
+              float2 zz = make_float2(v[2 * j], v[2 * j + 1]);
+              if constexpr (kHeads)
+                zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[2 * j], bb[2 * j + 1]));
+              const float2 a = __ffma2_rn(zz, make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
+              float e0 = ex2_approx(a.x);
+              float e1 = ex2_approx(a.y);
+              if (ragged) {
+                const int col = c * 32 + 2 * j;
+                e0 = col < ncols ? e0 : 0.f;
+                e1 = col + 1 < ncols ? e1 : 0.f;
+              }
+              sacc = __fadd2_rn(sacc, make_float2(e0, e1));
               if constexpr (kHeads) usum = fmaf(e0, v[2 * j], fmaf(e1, v[2 * j + 1], usum));
               p[j] = pack_bf16x2(e0, e1);
             }
@@ -478,6 +502,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (even) mbar_arrive(&tempty[acc]);
           else mbar_arrive_remote(tempty_even + acc * 8);
         }
+        const float ssum = sacc.x + sacc.y;
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
           if constexpr (kHeads) args.usum[static_cast<size_t>(nb) * args.M + row] = usum;
