@@ -336,34 +336,52 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const int y = (row_ok && args.targets) ? args.targets[row] : -1;
         const int yrel = y - n0;
         const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
-        float mx = -INFINITY, ssum = 0.f, zyv = 0.f;
+        float mx = -INFINITY, zyv = 0.f;
+        float2 sacc = make_float2(0.f, 0.f);    // sum of exp(z - mx), even and odd columns
         int amax = 0;
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
           float v[32];
           tmem_ld32(tbase + c * 32, v);
+          // the target logit, in the chunks holding some lane's target only
           const int yc = has_y ? yrel - c * 32 : -1;
-          float cm = -INFINITY;
-          int ci = 0;
+          if (__any_sync(0xffffffffu, static_cast<unsigned>(yc) < 32u)) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const bool in = c * 32 + j < ncols;
-            if (in && v[j] > cm) {          // strict: the first column reaching the max
-              cm = v[j];
-              ci = c * 32 + j;
-            }
-            zyv = (j == yc) ? v[j] : zyv;
+            for (int j = 0; j < 32; ++j) zyv = (j == yc) ? v[j] : zyv;
           }
-          if (cm > mx) {
-            ssum *= ex2_approx((mx - cm) * kLog2e);   // rescale to the new running max
-            mx = cm;
-            amax = ci;
+          if (c * 32 + 32 > ncols) {   // ragged last chunk (warp-uniform): columns
+                                       // past N neither win the max nor add to the sum
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (c * 32 + j >= ncols) v[j] = -INFINITY;
+          }
+          float t[11];
+#pragma unroll
+          for (int i = 0; i < 10; ++i) t[i] = fmax3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+          t[10] = fmaxf(v[30], v[31]);
+          const float cm = fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]),
+                                 fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
+          if (__any_sync(0xffffffffu, cm > mx)) {
+            int ci = 0;                           // the first column of the chunk holding cm
+#pragma unroll
+            for (int j = 31; j >= 0; --j) ci = (v[j] == cm) ? j : ci;
+            if (cm > mx) {                        // strict: an earlier equal maximum stays
+              const float f = ex2_approx((mx - cm) * kLog2e);   // rescale to the new max
+              sacc = make_float2(sacc.x * f, sacc.y * f);
+              mx = cm;
+              amax = c * 32 + ci;
+            }
           }
           const float mlog = mx * kLog2e;
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (c * 32 + j < ncols) ssum += ex2_approx(fmaf(v[j], kLog2e, -mlog));
+          for (int j = 0; j < 32; j += 2) {
+            const float2 a =
+                __ffma2_rn(make_float2(v[j], v[j + 1]), make_float2(kLog2e, kLog2e),
+                           make_float2(-mlog, -mlog));
+            sacc = __fadd2_rn(sacc, make_float2(ex2_approx(a.x), ex2_approx(a.y)));
+          }
         }
+        const float ssum = sacc.x + sacc.y;
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
@@ -419,7 +437,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           tmem_ld32(tbase + c * 32, v);
           if constexpr (kHeads) load_bias(c, bb);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) z[j] = kHeads ? fmaf(tau, v[j], bb[j]) : v[j];
+          for (int j = 0; j < 32; j += 2) {
+            if constexpr (kHeads) {
+              const float2 zz = __ffma2_rn(make_float2(tau, tau), make_float2(v[j], v[j + 1]),
+                                           make_float2(bb[j], bb[j + 1]));
+              z[j] = zz.x;
+              z[j + 1] = zz.y;
+            } else {
+              z[j] = v[j];
+              z[j + 1] = v[j + 1];
+            }
+          }
           // the target logit, in the chunks holding some lane's target only
           const int yc = has_y ? yrel - c * 32 : -1;
           if (__any_sync(0xffffffffu, static_cast<unsigned>(yc) < 32u)) {
@@ -445,7 +473,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const float mlog = mx * kLog2e;
         // the sum of exp(z - m) in two lanes of a packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
-        float usum = 0.f;
+        float2 uacc = make_float2(0.f, 0.f);   // kHeads: sum of exp(z - m) s, likewise
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
           if (lane == 0) bulk_wait_group_read<1>();
@@ -478,7 +506,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 e1 = col + 1 < ncols ? e1 : 0.f;
               }
               sacc = __fadd2_rn(sacc, make_float2(e0, e1));
-              if constexpr (kHeads) usum = fmaf(e0, v[2 * j], fmaf(e1, v[2 * j + 1], usum));
+              if constexpr (kHeads)
+                uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
               p[j] = pack_bf16x2(e0, e1);
             }
 #pragma unroll
@@ -505,7 +534,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const float ssum = sacc.x + sacc.y;
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
-          if constexpr (kHeads) args.usum[static_cast<size_t>(nb) * args.M + row] = usum;
+          if constexpr (kHeads)
+            args.usum[static_cast<size_t>(nb) * args.M + row] = uacc.x + uacc.y;
         }
         if constexpr (kHeads) {
           if (has_y) args.sy[row] = syv;
