@@ -93,12 +93,14 @@ def load_peaks():
 
 
 def strip_comments(src: str) -> str:
-    """C++ source without comments, blank lines or trailing spaces (string
-    literals in these files hold no comment markers)."""
+    """C++ source without comments, every run of whitespace made one space, so
+    that neither comments nor layout count as a change of the code (string
+    literals in these files hold no comment markers and no significant runs of
+    spaces)."""
     import re
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     src = re.sub(r"//[^\n]*", "", src)
-    return "\n".join(ln.rstrip() for ln in src.splitlines() if ln.strip())
+    return " ".join(src.split())
 
 
 def kernel_hash() -> str:

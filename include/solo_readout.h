@@ -100,8 +100,9 @@ typedef struct {
  * Bytes of device workspace one call with these dims needs (host-only; no
  * CUDA call).  The workspace holds the normalised inputs, the bf16
  * exponentials/gradient of the logits ([K*N, V]), per-token statistics,
- * fp32 partial tiles of the backward products and the flag word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims
- * out of range, SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0.
+ * fp32 partial tiles of the backward products and the flag word.  Returns
+ * SOLO_ERR_INVALID_ARG for NULL pointers or dims out of range,
+ * SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0.
  */
 solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
 

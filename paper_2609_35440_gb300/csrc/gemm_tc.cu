@@ -497,7 +497,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               float2 zz = make_float2(v[2 * j], v[2 * j + 1]);
               if constexpr (kHeads)
                 zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[2 * j], bb[2 * j + 1]));
-              const float2 a = __ffma2_rn(zz, make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
+              const float2 a =
+                  __ffma2_rn(zz, make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
               float e0 = ex2_approx(a.x);
               float e1 = ex2_approx(a.y);
               if (ragged) {
