@@ -414,10 +414,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         // warp's vector loads hit the same addresses
         const bool bias_vec = (args.V & 3) == 0;
         auto load_bias = [&](int c, float (&b)[32]) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) b[j] = 0.f;
-          if (!kHeads || brow == nullptr) return;
-          if (bias_vec && c * 32 + 32 <= ncols) {
+          if (brow != nullptr && bias_vec && c * 32 + 32 <= ncols) {
+            // the common case: eight 16-byte loads fill every value
             const float4* b4 = reinterpret_cast<const float4*>(brow + c * 32);
 #pragma unroll
             for (int q4 = 0; q4 < 8; ++q4) {
@@ -427,7 +425,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           } else {
 #pragma unroll
             for (int j = 0; j < 32; ++j)
-              if (c * 32 + j < ncols) b[j] = __ldg(brow + c * 32 + j);
+              b[j] = (brow != nullptr && c * 32 + j < ncols) ? __ldg(brow + c * 32 + j) : 0.f;
           }
         };
         float mx = -INFINITY, zyv = 0.f, syv = 0.f;

@@ -19,8 +19,10 @@ BASE_KEYS = {"metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_ste
 
 
 def _run(*args, timeout=600) -> dict:
-    out = subprocess.run([sys.executable, "bench.py", *args], cwd=ROOT, check=True,
-                         capture_output=True, text=True, timeout=timeout).stdout
+    proc = subprocess.run([sys.executable, "bench.py", *args], cwd=ROOT, capture_output=True,
+                          text=True, timeout=timeout)
+    assert proc.returncode == 0, proc.stderr[-4000:]
+    out = proc.stdout
     lines = [ln for ln in out.splitlines() if ln.startswith("{")]
     assert len(lines) == 1, out          # exactly one JSON line on stdout
     return json.loads(lines[0])
@@ -34,6 +36,15 @@ def _check_base(j: dict, steps: int, warmup: int):
     assert j["scaling"] in ("weak", "strong")
     assert j["config"]["workload"] == SMALL
     assert j["vs_baseline"] is None
+
+
+def test_cpu_baseline_sample_stays_within_the_workload():
+    sys.path.insert(0, ROOT)
+    import bench
+    wl = bench.workload_from_name(SMALL)
+    cb = bench.cpu_baseline(wl, 0.5)
+    rows = int(cb["sample"].split()[1])          # "first <rows> tokens of each ..."
+    assert cb["value"] > 0 and 1 <= rows <= wl.N
 
 
 def test_reference_arm_line():
@@ -52,6 +63,7 @@ def test_default_arm_line():
     j = _run("--steps", "3", "--warmup", "3", "--workload", SMALL, "--cpu-seconds", "1")
     _check_base(j, 3, 3)
     assert j["dtype"] == "bf16" and j["data"] == "synthetic"
+    assert "not a reportable configuration" in j["config"]["l2"]   # 1 MB of inputs
     r = j["roofline"]
     assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
     assert r["achieved"] > 0 and r["peak"] > 0
