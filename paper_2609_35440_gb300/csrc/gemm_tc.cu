@@ -121,6 +121,119 @@ __device__ __forceinline__ bool mbar_wait_hw(uint64_t* bar, uint32_t parity, vol
   return mbar_wait(bar, parity, abort);
 }
 
+// ---- the RMSNorm backward, fused into the dX̂ epilogue -----------------------
+// Eq. 3 sends delta_k back through the final RMSNorm.  With dxhat = G W,
+//   dh_j = r gamma_j dxhat_j - (r^3 / d) h_j S,   S = sum_l gamma_l h_l dxhat_l.
+// S needs a whole row of dxhat, which one 256-column tile does not hold.  But
+// gamma_l h_l r is xhat_l before its bf16 rounding, so
+//   S = (1/r) sum_l xhat_l dxhat_l = (1/r) sum_v G_v s_v
+//     = tau inv_nvalid (E_p[s] - s_y) / r
+// (s = W xhat, the logits before temperature and bias), which the logits
+// epilogue and the log-sum-exp pass reduce per row (edz).  The two forms
+// differ only by xhat's rounding, far inside the gradient tolerances.
+
+struct NormRow {
+  bool ok;             // a row of the product
+  bool dg;             // a row of the final module (its dgamma terms are summed)
+  float r, coef;       // r_i and (r_i^3 / d) S_i
+  const uint16_t* h;   // the row of hidden (bf16)
+  uint16_t* dh;        // the row of dhidden (bf16)
+};
+
+__device__ __forceinline__ NormRow norm_row(const GemmArgs& g, int64_t row) {
+  NormRow nr{false, false, 0.f, 0.f, nullptr, nullptr};
+  if (row >= g.M) return nr;
+  const int k = static_cast<int>(row / g.tokens_per_module);
+  if (!in_bounds(k < g.modules, g.flags)) return nr;
+  const int64_t n = row - static_cast<int64_t>(k) * g.tokens_per_module;
+  const float r = g.r[row];
+  const float tau = g.tau ? g.tau[k] : 1.f;
+  nr.ok = true;
+  nr.dg = g.dg_part != nullptr && row >= g.dg_row0;
+  nr.r = r;
+  nr.coef = r * r * (tau * g.inv_nvalid[k] * g.edz[row]) / static_cast<float>(g.N);
+  nr.h = g.hidden[k] + n * g.N;
+  nr.dh = g.dhidden[k] + n * g.N;
+  return nr;
+}
+
+// Sum over the warp's lanes of p[j], for every j at once: after five halving
+// exchanges lane j holds the sum of p[j] (31 shuffles, fixed order).
+__device__ __forceinline__ float reduce_scatter32(float (&p)[32]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 0; s < 5; ++s) {
+    const int o = 16 >> s;                   // partner distance = values kept
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i < o) {
+        const float send = upper ? p[i] : p[i + o];
+        const float keep = upper ? p[i + o] : p[i];
+        p[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      }
+    }
+  }
+  return p[0];
+}
+
+// Columns [col0, col0 + 32) of this lane's row, cols of them valid (a multiple
+// of 8), dxhat in v: dH in bf16, and, when the warp holds rows of the final
+// module (dg_warp, warp-uniform), the column sums over its 32 rows of
+// dxhat h r, lane j storing column col0 + j at dg_dst[j].
+__device__ __forceinline__ void norm_bwd_chunk(const GemmArgs& g, const float (&v)[32], int col0,
+                                               int cols, const NormRow& nr, bool dg_warp,
+                                               float* dg_dst) {
+  const int lane = threadIdx.x & 31;
+  float h[32], gm[32];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint4 hv = make_uint4(0, 0, 0, 0), gv = make_uint4(0, 0, 0, 0);
+    if (8 * q < cols) {
+      gv = __ldg(reinterpret_cast<const uint4*>(g.gamma + col0) + q);
+      if (nr.ok) hv = __ldg(reinterpret_cast<const uint4*>(nr.h + col0) + q);
+    }
+    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w}, gw[4] = {gv.x, gv.y, gv.z, gv.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      h[8 * q + 2 * j] = __uint_as_float(hw[j] << 16);
+      h[8 * q + 2 * j + 1] = __uint_as_float(hw[j] & 0xFFFF0000u);
+      gm[8 * q + 2 * j] = __uint_as_float(gw[j] << 16);
+      gm[8 * q + 2 * j + 1] = __uint_as_float(gw[j] & 0xFFFF0000u);
+    }
+  }
+  if (nr.ok) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (8 * q < cols) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int c = 8 * q + 2 * j;
+          w[j] = pack_bf16x2(fmaf(nr.r * gm[c], v[c], -nr.coef * h[c]),
+                             fmaf(nr.r * gm[c + 1], v[c + 1], -nr.coef * h[c + 1]));
+        }
+        reinterpret_cast<uint4*>(nr.dh + col0)[q] = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
+  }
+  if (dg_warp) {
+    float p[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) p[j] = nr.dg ? v[j] * h[j] * nr.r : 0.f;
+    const float sum = reduce_scatter32(p);
+    if (dg_dst != nullptr && lane < cols) dg_dst[lane] = sum;
+  }
+}
+
+// The dgamma partial row of the 32-row block starting at row_base (a multiple
+// of 32), for columns from col0; null when the block holds no final-module row.
+__device__ __forceinline__ float* dg_block(const GemmArgs& g, int64_t row_base, int col0) {
+  const int64_t rb = (row_base >> 5) - (g.dg_row0 >> 5);
+  if (g.dg_part == nullptr || !in_bounds(rb >= 0 && rb < g.dg_blocks, g.flags)) return nullptr;
+  return g.dg_part + rb * g.N + col0;
+}
+
 __device__ __forceinline__ void spin_ns(uint64_t ns) {
   const uint64_t t0 = globaltimer_ns();
   while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
@@ -471,7 +584,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const float mlog = mx * kLog2e;
         // the sum of exp(z - m) in two lanes of a packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
-        float2 uacc = make_float2(0.f, 0.f);   // kHeads: sum of exp(z - m) s, likewise
+        float2 uacc = make_float2(0.f, 0.f);   // sum of exp(z - m) s, likewise
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
           if (lane == 0) bulk_wait_group_read<1>();
@@ -505,8 +618,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 e1 = col + 1 < ncols ? e1 : 0.f;
               }
               sacc = __fadd2_rn(sacc, make_float2(e0, e1));
-              if constexpr (kHeads)
-                uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
+              uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
               p[j] = pack_bf16x2(e0, e1);
             }
 #pragma unroll
@@ -533,13 +645,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const float ssum = sacc.x + sacc.y;
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
-          if constexpr (kHeads)
-            args.usum[static_cast<size_t>(nb) * args.M + row] = uacc.x + uacc.y;
+          args.usum[static_cast<size_t>(nb) * args.M + row] = uacc.x + uacc.y;
         }
         if constexpr (kHeads) {
           if (has_y) args.sy[row] = syv;
         }
         if (has_y) args.zy[row] = zyv;
+      } else if (MODE == kDxhat && args.norm_fused && t < args.full_tiles) {
+        // whole dX̂ tile: the RMSNorm backward straight from TMEM to bf16 dH
+        const NormRow nr = norm_row(args, row);
+        const bool dg_warp = __any_sync(0xffffffffu, nr.dg);
+        float* dg = dg_warp ? dg_block(args, m0 + 32 * q, n0) : nullptr;
+        for (int c = 0; c < kBN / 32; ++c) {
+          if (c * 32 >= ncols) break;
+          float v[32];
+          tmem_ld32(tbase + c * 32, v);
+          norm_bwd_chunk(args, v, n0 + c * 32, min(32, ncols - c * 32), nr, dg_warp,
+                         dg ? dg + c * 32 : nullptr);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (even) mbar_arrive(&tempty[acc]);
+          else mbar_arrive_remote(tempty_even + acc * 8);
+        }
       } else {
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
@@ -659,7 +788,44 @@ __global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, floa
   }
 }
 
+// kDxhat with norm_fused: the RMSNorm backward of the cut tiles, from their
+// fp32 dX̂ summed by split_fixup_kernel.  Grid (cut tiles, 8 blocks of 32
+// rows); warp w handles the tile's columns [32 w, 32 w + 32), lane i row i.
+__global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, const float* dxhat) {
+  const int t = g.full_tiles + static_cast<int>(blockIdx.x);
+  int mb, nb;
+  tile_coords(t, g, mb, nb);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t row_base = static_cast<int64_t>(mb) * kPairRows + blockIdx.y * 32;
+  const int64_t row = row_base + lane;
+  const int col0 = nb * kBN + warp * 32;
+  if (col0 >= g.N) return;                       // warp-uniform
+  const int cols = min(32, g.N - col0);
+  const NormRow nr = norm_row(g, row);
+  float v[32];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (nr.ok && 4 * q < cols)
+      x = *reinterpret_cast<const float4*>(dxhat + row * g.N + col0 + 4 * q);
+    v[4 * q] = x.x;
+    v[4 * q + 1] = x.y;
+    v[4 * q + 2] = x.z;
+    v[4 * q + 3] = x.w;
+  }
+  const bool dg_warp = __any_sync(0xffffffffu, nr.dg);
+  norm_bwd_chunk(g, v, col0, cols, nr, dg_warp, dg_warp ? dg_block(g, row_base, col0) : nullptr);
+}
+
 }  // namespace
+
+cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* dxhat, cudaStream_t stream) {
+  const int cut = g.num_tiles - g.full_tiles;
+  if (!g.norm_fused || g.split < 2 || cut <= 0) return cudaSuccess;
+  cut_tiles_norm_kernel<<<dim3(cut, kPairRows / 32), 256, 0, stream>>>(g, dxhat);
+  return launched();
+}
 
 cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const float* aux,
                                cudaStream_t stream) {

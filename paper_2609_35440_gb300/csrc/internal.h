@@ -49,11 +49,14 @@ constexpr int kStages = 6 * 64 / kBK;      // 192 KB of operand ring per CTA
 constexpr int kKAtoms = kBK / 64;          // 128-byte swizzle atoms along K per row
 constexpr int kGemmThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: epilogue
 
+constexpr int kMaxModules = 16;
+
 // The products of the GEMM kernel.
 enum GemmMode : int {
   kLogits = 0,  // Z = Xhat W^T (A: Xhat K-major, B: W K-major); epilogue: per-tile
                 //   max / sum of exp, target logit, bf16 exp(z - tile max) stored
-  kDxhat = 1,   // dXhat = G W (A: G K-major, B: W MN-major); epilogue: fp32 store
+  kDxhat = 1,   // dXhat = G W (A: G K-major, B: W MN-major); epilogue: the RMSNorm
+                //   backward into bf16 dH (norm_fused), or fp32 dXhat
   kDW = 2,      // dW = G^T Xhat over the final module (A: G MN-major,
                 //   B: Xhat MN-major); epilogue: fp32 store
   kExit = 3,    // Z = Xhat W^T for decoding only; epilogue: per-tile max, sum of
@@ -94,6 +97,20 @@ struct GemmArgs {
   int64_t tokens_per_module;
   float* usum;             // [n_blocks, M]: sum over the tile of exp(z - m) * s
   float* sy;               // [M]: s at the target (before temperature and bias)
+  // kDxhat with the RMSNorm backward fused into the epilogue (norm_fused = 1):
+  // whole tiles write dH = r gamma dxhat - (r^3 / d) h S in bf16 and the final
+  // module's dgamma partial sums; cut tiles store fp32 dXhat as without it.
+  int32_t norm_fused;
+  int32_t modules;                       // K
+  const uint16_t* hidden[kMaxModules];   // [N, d] bf16 per module
+  uint16_t* dhidden[kMaxModules];        // [N, d] bf16 per module
+  const uint16_t* gamma;                 // [d]
+  const float* r;                        // [M]
+  const float* edz;                      // [M]: E_p[s] - s_y of a kept token, else 0
+  const float* inv_nvalid;               // [K]
+  float* dg_part;          // [dg_blocks, d] or null: per 32-row block of the final module
+  int32_t dg_blocks;
+  int64_t dg_row0;         // first row of the final module
 };
 
 size_t gemm_smem_bytes();
@@ -121,10 +138,11 @@ cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& 
 // out (fp32, row stride ld) += the auxiliary parts of every cut tile.
 cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const float* aux,
                                cudaStream_t stream);
+// kDxhat with norm_fused, after launch_split_fixup: the RMSNorm backward (dH,
+// dgamma partials) of the cut tiles, from their summed fp32 dXhat.
+cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* dxhat, cudaStream_t stream);
 
 // ---- row kernels ---------------------------------------------------------------
-
-constexpr int kMaxModules = 16;
 
 struct RowArgs {
   const uint16_t* hidden[kMaxModules];
@@ -144,6 +162,8 @@ struct RowArgs {
   uint16_t* xhat;       // [M, d]
   float* lse;           // [M]
   float* zy;            // [M]
+  float* edz;           // [M]: E_p[s] - s_y per kept token (0 if masked), for the
+                        //      RMSNorm backward's row sum
   float2* stats;        // [n_tiles_v, M]
   double* part_sum;     // [K, part_blocks]
   int32_t* part_cnt;    // [K, part_blocks]
@@ -152,10 +172,8 @@ struct RowArgs {
   float* loss_tok;      // [K, N] or null
   float* loss_mean;     // [K]
   uint16_t* P;          // [M, ldp] bf16: exp(z - tile max), turned into G in place
-  float* dxhat;         // [M, d]
-  float* dgamma_part;   // [dg_chunks, d]
+  float* dgamma_part;   // [dg_chunks, d]: per 32-row block of the final module
   int32_t dg_chunks;
-  int32_t dg_rows;      // rows per dgamma chunk
   float* dgamma;        // [d] or null
   uint32_t* flags;
   // exit readout
@@ -182,7 +200,6 @@ cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads = false);
 cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s);
 // G in place; with a.dbias also the per-module column sums of dL/dz.
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s);
-cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts);
 cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s);
 
 }  // namespace solo

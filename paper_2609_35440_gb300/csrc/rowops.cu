@@ -1,6 +1,7 @@
-// Row-wise kernels of the readout path: the final RMSNorm and its backward,
-// the log-sum-exp combination of per-tile statistics with the token loss and
-// module means, the gradient of the logits, and the dgamma reduction.
+// Row-wise kernels of the readout path: the final RMSNorm, the log-sum-exp
+// combination of per-tile statistics with the token loss and module means, the
+// gradient of the logits, and the dgamma reduction.  (The RMSNorm backward runs
+// in the epilogue of the dX̂ GEMM.)
 //
 // All reductions run in a fixed order (no floating-point atomics), so every
 // output is bitwise reproducible from run to run.
@@ -25,12 +26,6 @@ __device__ __forceinline__ void unpack8(const uint4& x, float (&f)[8]) {
   f[2] = bf16_lo(x.y); f[3] = bf16_hi(x.y);
   f[4] = bf16_lo(x.z); f[5] = bf16_hi(x.z);
   f[6] = bf16_lo(x.w); f[7] = bf16_hi(x.w);
-}
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
 }
 
 __device__ __forceinline__ bool token_kept(const RowArgs& a, int64_t row, int y) {
@@ -233,7 +228,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       for (int u = 0; u < 8; ++u) {       // independent loads, issued together
         const bool in = t0 + u < a.n_tiles_v;
         st[u] = in ? a.stats[static_cast<int64_t>(t0 + u) * M + row] : make_float2(-INFINITY, 0.f);
-        if constexpr (kHeads) uu[u] = in ? a.usum[static_cast<int64_t>(t0 + u) * M + row] : 0.f;
+        if constexpr (!kExit) uu[u] = in ? a.usum[static_cast<int64_t>(t0 + u) * M + row] : 0.f;
       }
       float cm = mx;
 #pragma unroll
@@ -243,12 +238,12 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       }
       const float rescale = expf(mx - cm);  // mx = -inf only before the first tile (s = 0)
       s *= rescale;
-      if constexpr (kHeads) us *= rescale;
+      if constexpr (!kExit) us *= rescale;
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const float f = expf(st[u].x - cm);
         s += st[u].y * f;
-        if constexpr (kHeads) us += uu[u] * f;
+        if constexpr (!kExit) us += uu[u] * f;
       }
       mx = cm;
     }
@@ -267,7 +262,14 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     if (a.loss_tok) a.loss_tok[row] = loss;
     lsum = loss;
     cnt = kept ? 1 : 0;
-    if constexpr (kHeads) tsum = kept ? static_cast<double>(us / s - a.sy[row]) : 0.0;
+    if constexpr (!kExit) {
+      // E_p[s] - s_y (s: the logits before temperature and bias; s = z
+      // without them): the temperature's gradient term and, scaled, the
+      // RMSNorm backward's row sum
+      const float e = kept ? us / s - (kHeads ? a.sy[row] : a.zy[row]) : 0.f;
+      a.edz[row] = e;
+      if constexpr (kHeads) tsum = e;
+    }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(a.flags, SOLO_FLAG_BAD_TARGET);
   __shared__ double ssum[8], stau[8];
@@ -464,103 +466,39 @@ __global__ void __launch_bounds__(256) dbias_reduce_kernel(const RowArgs a) {
   a.dbias[static_cast<int64_t>(k) * a.V + v] = acc;
 }
 
-// ---- RMSNorm backward: dh = r gamma dxhat - (r^3/d) h sum_l gamma_l dxhat_l h_l --
+// ---- dgamma of the final module: the fixed-order sum of the partial sums per
+// 32-row block that the RMSNorm backward (fused into the dX̂ GEMM) wrote -----
 
-template <int VPL>
-__global__ void __launch_bounds__(256) norm_bwd_kernel(const RowArgs a) {
-  const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  const int lane = threadIdx.x & 31;
-  const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
-  if (row >= M) return;
-  const int k = static_cast<int>(row / a.N);
-  const int64_t n = row - static_cast<int64_t>(k) * a.N;
-  const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
-  const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
-  const float4* dx = reinterpret_cast<const float4*>(a.dxhat + row * a.d);
-  const int nv = a.d / 8;
-  constexpr int kCache = VPL > 0 ? VPL : 1;
-  uint4 hc[kCache];
-  float4 d0c[kCache], d1c[kCache];
-  float c = 0.f;
-  auto dot = [&](const uint4& hx, const uint4& gx, const float4& d0, const float4& d1) {
-    float f[8], gg[8];
-    unpack8(hx, f);
-    unpack8(gx, gg);
-    c = fmaf(gg[0] * d0.x, f[0], c); c = fmaf(gg[1] * d0.y, f[1], c);
-    c = fmaf(gg[2] * d0.z, f[2], c); c = fmaf(gg[3] * d0.w, f[3], c);
-    c = fmaf(gg[4] * d1.x, f[4], c); c = fmaf(gg[5] * d1.y, f[5], c);
-    c = fmaf(gg[6] * d1.z, f[6], c); c = fmaf(gg[7] * d1.w, f[7], c);
-  };
-  if constexpr (VPL > 0) {
-    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int u = 0; u < VPL; ++u) {
-      const int v = lane + 32 * u;
-      const bool in = v < nv;
-      hc[u] = in ? __ldg(h + v) : make_uint4(0, 0, 0, 0);
-      d0c[u] = in ? dx[2 * v] : z4;
-      d1c[u] = in ? dx[2 * v + 1] : z4;
-    }
-#pragma unroll
-    for (int u = 0; u < VPL; ++u) {
-      const int v = lane + 32 * u;
-      if (v < nv) dot(hc[u], __ldg(g + v), d0c[u], d1c[u]);
-    }
-  } else {
-    for (int v = lane; v < nv; v += 32) dot(__ldg(h + v), __ldg(g + v), dx[2 * v], dx[2 * v + 1]);
-  }
-  c = warp_sum(c);
-  const float r = a.r[row];
-  const float coef = r * r * r * c / static_cast<float>(a.d);
-  uint4* out = reinterpret_cast<uint4*>(a.dhidden[k] + n * a.d);
-  auto emit = [&](int v, const uint4& hx, const float4& d0, const float4& d1) {
-    float f[8], gg[8];
-    unpack8(hx, f);
-    unpack8(__ldg(g + v), gg);
-    const float dd[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
-    float o[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) o[j] = fmaf(r * gg[j], dd[j], -coef * f[j]);
-    out[v] = make_uint4(pack2(o[0], o[1]), pack2(o[2], o[3]), pack2(o[4], o[5]), pack2(o[6], o[7]));
-  };
-  if constexpr (VPL > 0) {
-#pragma unroll
-    for (int u = 0; u < VPL; ++u) {
-      const int v = lane + 32 * u;
-      if (v < nv) emit(v, hc[u], d0c[u], d1c[u]);
-    }
-  } else {
-    for (int v = lane; v < nv; v += 32) emit(v, __ldg(h + v), dx[2 * v], dx[2 * v + 1]);
-  }
-}
-
-// ---- dgamma of the final module: sum_i dxhat_ij h_ij r_i, two fixed-order stages --
-
-__global__ void __launch_bounds__(256) dgamma_part_kernel(const RowArgs a) {
-  const int j = blockIdx.x * 256 + threadIdx.x;
-  const int chunk = blockIdx.y;
-  if (j >= a.d) return;
-  const int k = a.K - 1;
-  const int64_t n0 = static_cast<int64_t>(chunk) * a.dg_rows;
-  const int64_t n1 = min(a.N, n0 + a.dg_rows);
-  const uint16_t* h = a.hidden[k];
-  const int64_t row0 = static_cast<int64_t>(k) * a.N;
-  if (!in_bounds(chunk < a.dg_chunks && row0 + n1 <= static_cast<int64_t>(a.K) * a.N, a.flags))
-    return;
-  float acc = 0.f;
-  for (int64_t n = n0; n < n1; ++n) {
-    const float hv = __uint_as_float(static_cast<uint32_t>(h[n * a.d + j]) << 16);
-    acc = fmaf(a.dxhat[(row0 + n) * a.d + j] * a.r[row0 + n], hv, acc);
-  }
-  a.dgamma_part[static_cast<int64_t>(chunk) * a.d + j] = acc;
-}
-
+// One CTA per 32 columns: warp w sums a fixed segment of the partial rows for
+// its 32 columns (lane = column, 128-byte rows), then warp 0 adds the eight
+// segment sums in order.
 __global__ void __launch_bounds__(256) dgamma_reduce_kernel(const RowArgs a) {
-  const int j = blockIdx.x * 256 + threadIdx.x;
-  if (j >= a.d) return;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int j = blockIdx.x * 32 + lane;
+  const int seg = (a.dg_chunks + 7) / 8;
+  const int c1 = min(a.dg_chunks, (warp + 1) * seg);
   float acc = 0.f;
-  for (int c = 0; c < a.dg_chunks; ++c) acc += a.dgamma_part[static_cast<int64_t>(c) * a.d + j];
-  a.dgamma[j] = acc;
+  if (j < a.d) {
+    int c = warp * seg;
+    for (; c + 8 <= c1; c += 8) {          // eight loads in flight, added in order
+      float x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = a.dgamma_part[static_cast<int64_t>(c + u) * a.d + j];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc += x[u];
+    }
+    for (; c < c1; ++c) acc += a.dgamma_part[static_cast<int64_t>(c) * a.d + j];
+  }
+  __shared__ float seg_sum[8][32];
+  seg_sum[warp][lane] = acc;
+  __syncthreads();
+  if (warp == 0 && j < a.d) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += seg_sum[w][lane];
+    a.dgamma[j] = t;
+  }
 }
 
 }  // namespace
@@ -626,24 +564,8 @@ cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
   return launched();
 }
 
-cudaError_t launch_norm_bwd(const RowArgs& a, cudaStream_t s, bool want_dgamma_parts) {
-  const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  const unsigned grid = static_cast<unsigned>((M + 7) / 8);
-  switch (vectors_per_lane(a.d)) {
-    case 1: norm_bwd_kernel<1><<<grid, 256, 0, s>>>(a); break;
-    case 2: norm_bwd_kernel<2><<<grid, 256, 0, s>>>(a); break;
-    case 4: norm_bwd_kernel<4><<<grid, 256, 0, s>>>(a); break;
-    case 8: norm_bwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
-    default: norm_bwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
-  }
-  cudaError_t e = launched();
-  if (e != cudaSuccess || !want_dgamma_parts) return e;
-  dgamma_part_kernel<<<dim3((a.d + 255) / 256, a.dg_chunks), 256, 0, s>>>(a);
-  return launched();
-}
-
 cudaError_t launch_dgamma_reduce(const RowArgs& a, cudaStream_t s) {
-  dgamma_reduce_kernel<<<(a.d + 255) / 256, 256, 0, s>>>(a);
+  dgamma_reduce_kernel<<<(a.d + 31) / 32, 256, 0, s>>>(a);
   return launched();
 }
 

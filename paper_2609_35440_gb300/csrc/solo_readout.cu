@@ -7,8 +7,10 @@
 //                sum of exp, target logit, bf16 exp(z - tile max)  [K*N, V]
 //   lse          log-sum-exp per row, token loss, module means, 1/Nvalid
 //   grad         (softmax - onehot)/Nvalid in place, bf16        [K*N, V]
-//   dxhat        tensor-core G W, fp32                            [K*N, d]
-//   norm_bwd     dH through the RMSNorm Jacobian, dgamma partial sums
+//   dxhat        tensor-core G W with the RMSNorm backward in its epilogue:
+//                bf16 dH and the final module's dgamma partial sums [K*N, d]
+//   norm_bwd     the same for the tiles whose last wave was cut along V
+//                (their fp32 dXhat summed first)
 //   dW           tensor-core G^T xhat over the final module       [V, d]
 //   dgamma       fixed-order sum of the partials                  [d]
 #include <cudaTypedefs.h>
@@ -38,7 +40,6 @@ namespace {
 using namespace solo;
 
 constexpr size_t kAlign = 1024;
-constexpr int kDgRows = 64;
 // Tile raster (in 256-row pair blocks) per product, from a sweep on GB300.
 constexpr int kGroupLogits = 16;
 constexpr int kGroupDxhat = 4;
@@ -53,7 +54,7 @@ struct Layout {
   int part_blocks = 0;
   int dg_chunks = 0;
   int db_chunks = 0;
-  size_t flags = 0, r = 0, lse = 0, zy = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
+  size_t flags = 0, r = 0, lse = 0, zy = 0, edz = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
   size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
   int aux_slots = 0;
@@ -78,7 +79,9 @@ Layout make_layout(const solo_dims_t& d) {
   L.ldp = static_cast<int>(align_up(d.V, 8));
   L.n_tiles_v = (d.V + kBN - 1) / kBN;
   L.part_blocks = static_cast<int>((d.N + 255) / 256);
-  L.dg_chunks = static_cast<int>((d.N + kDgRows - 1) / kDgRows);
+  // dgamma partial sums per 32-row block holding rows of the final module
+  const int64_t row0_final = static_cast<int64_t>(d.K - 1) * d.N;
+  L.dg_chunks = static_cast<int>(((L.M - 1) >> 5) - (row0_final >> 5) + 1);
   L.db_chunks = static_cast<int>((d.N + kGradRows - 1) / kGradRows);
   const size_t M = static_cast<size_t>(L.M);
   size_t off = 0;
@@ -91,6 +94,7 @@ Layout make_layout(const solo_dims_t& d) {
   L.r = take(M * 4);
   L.lse = take(M * 4);
   L.zy = take(M * 4);
+  L.edz = take(M * 4);
   L.part_sum = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
   L.part_cnt = take(static_cast<size_t>(d.K) * L.part_blocks * 4);
   L.inv_nvalid = take(SOLO_MAX_MODULES * 4);
@@ -291,6 +295,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.xhat = reinterpret_cast<uint16_t*>(ws + L.xhat);
   ra.lse = reinterpret_cast<float*>(ws + L.lse);
   ra.zy = reinterpret_cast<float*>(ws + L.zy);
+  ra.edz = reinterpret_cast<float*>(ws + L.edz);
   ra.stats = reinterpret_cast<float2*>(ws + L.stats);
   ra.part_sum = reinterpret_cast<double*>(ws + L.part_sum);
   ra.part_cnt = reinterpret_cast<int32_t*>(ws + L.part_cnt);
@@ -299,10 +304,9 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.loss_tok = loss_tok;
   ra.loss_mean = loss_mean;
   ra.P = reinterpret_cast<uint16_t*>(ws + L.P);
-  ra.dxhat = reinterpret_cast<float*>(ws + L.dxhat);
+  float* dxhat = reinterpret_cast<float*>(ws + L.dxhat);
   ra.dgamma_part = reinterpret_cast<float*>(ws + L.dgp);
   ra.dg_chunks = L.dg_chunks;
-  ra.dg_rows = kDgRows;
   ra.dgamma = dgamma;
   ra.flags = reinterpret_cast<uint32_t*>(ws + L.flags);
   ra.tau = tau;
@@ -329,7 +333,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
             make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
             make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBM) &&
             make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK) &&
-            make_map(&mDX, F32, ra.dxhat, d, M, d * 4, 32, 32);
+            make_map(&mDX, F32, dxhat, d, M, d * 4, 32, 32);
   if (ok && dW) {
     ok = make_map(&mG_mn, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBK) &&
          make_map(&mX_mn, BF, ra.xhat, d, M, d * 2, 64, kBK) &&
@@ -384,13 +388,27 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
   gx.group_m = kGroupDxhat;
   gx.num_tiles = gx.m_blocks * gx.n_blocks;
+  // the RMSNorm backward in the epilogue (dH, and dgamma partials when wanted)
+  gx.norm_fused = 1;
+  gx.modules = D.K;
+  for (int k = 0; k < D.K; ++k) {
+    gx.hidden[k] = ra.hidden[k];
+    gx.dhidden[k] = ra.dhidden[k];
+  }
+  gx.gamma = ra.gamma;
+  gx.r = ra.r;
+  gx.edz = ra.edz;
+  gx.inv_nvalid = ra.inv_nvalid;
+  gx.dg_part = dgamma ? ra.dgamma_part : nullptr;
+  gx.dg_blocks = L.dg_chunks;
+  gx.dg_row0 = static_cast<int64_t>(D.K - 1) * D.N;
   plan_units(gx, sms, true);
   if (!mark(SOLO_STAGE_DXHAT) ||
       fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, mAux, gx, sms, stream)) ||
-      fail(launch_split_fixup(gx, ra.dxhat, D.d, aux, stream)))
+      fail(launch_split_fixup(gx, dxhat, D.d, aux, stream)))
     return SOLO_ERR_CUDA;
 
-  if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_norm_bwd(ra, stream, dgamma != nullptr)))
+  if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_cut_tiles_norm(gx, dxhat, stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_DW)) return SOLO_ERR_CUDA;
