@@ -80,8 +80,11 @@ enum {
   SOLO_STAGE_LOGITS = 1,    /* tensor-core X W^T, per-tile max/sum, exps    */
   SOLO_STAGE_LSE = 2,       /* logsumexp, token loss, module means          */
   SOLO_STAGE_GRAD = 3,      /* dL/dz = (softmax - onehot) / Nvalid, bf16    */
-  SOLO_STAGE_DXHAT = 4,     /* tensor-core dXhat = G W                      */
-  SOLO_STAGE_NORM_BWD = 5,  /* dH through the RMSNorm Jacobian, dgamma parts */
+  SOLO_STAGE_DXHAT = 4,     /* tensor-core dXhat = G W; its epilogue takes
+                               dH through the RMSNorm Jacobian and forms the
+                               dgamma partial sums                           */
+  SOLO_STAGE_NORM_BWD = 5,  /* the same for the few tiles whose reduction
+                               was cut into parts (after their fix-up)       */
   SOLO_STAGE_DW = 6,        /* tensor-core dW = G^T Xhat, final module      */
   SOLO_STAGE_DGAMMA = 7,    /* dgamma reduction, final module               */
   SOLO_NUM_STAGES = 8

@@ -25,12 +25,15 @@
 //
 // Epilogues:
 //  kLogits  Z = Xhat W^T.  Per row and 256-column tile: m = max_v z,
-//           s = sum_v exp(z - m), the target logit when the target falls in the
-//           tile, and the bf16 values exp(z - m) written to a [rows, V] buffer
-//           with TMA stores.  These feed the log-sum-exp of the cross-entropy
-//           (Eq. 2 and the local loss of Algorithm 1) and, rescaled, its
+//           s = sum_v exp(z - m), sum_v exp(z - m) z, the target logit when
+//           the target falls in the tile, and the bf16 values exp(z - m)
+//           written to a [rows, V] buffer with TMA stores.  These feed the
+//           log-sum-exp of the cross-entropy (Eq. 2 and the local loss of
+//           Algorithm 1), the RMSNorm backward's row sum and, rescaled, the
 //           gradient, so the logits are never written and never recomputed.
-//  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3; fp32 out.
+//  kDxhat   dXhat = G W, the readout factor W^T delta_k of Eq. 3, and in the
+//           same epilogue the final RMSNorm's backward: bf16 dH and the final
+//           module's dgamma partial sums (fp32 dXhat for the cut tiles).
 //  kDW      dW = G^T Xhat over the final module's tokens; fp32 out.
 //  kLogitsHeads  as kLogits with each head's temperature and bias (Algorithm
 //           1: z = tau_k W-bar xhat + b_k), plus per tile sum exp(z - m) s and
