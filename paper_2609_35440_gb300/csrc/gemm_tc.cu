@@ -587,7 +587,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         const float mlog = mx * kLog2e;
         // the sum of exp(z - m) in two lanes of a packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
-        float2 uacc = make_float2(0.f, 0.f);   // sum of exp(z - m) s, likewise
+        // sum of exp(z - m) (s - c), likewise, with c = m / tau: near the tile
+        // maximum s - c is small, so a confident row's E_p[s] - s_y keeps its
+        // relative precision (the log-sum-exp pass adds (c - s_y) times the
+        // sum of exp back per tile, with the same c)
+        const float cs = tau != 0.f ? mx / tau : 0.f;
+        float2 uacc = make_float2(0.f, 0.f);
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
           if (lane == 0) bulk_wait_group_read<1>();
@@ -606,6 +611,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             }
             uint32_t p[16];
             const bool ragged = c * 32 + 32 > ncols;      // warp-uniform
+            // The target's own term is left out of the tile's sums (the
+            // stored exponential keeps it): the log-sum-exp pass then forms
+            // lse - z_y = log1p(sum over v != y of exp(z_v - z_y)), and 1 - p_y
+            // and E_p[s] - s_y of a confident row do not cancel.
+            const int ycol = has_y ? yrel - c * 32 : -1;
+            const bool tgt = __any_sync(0xffffffffu, static_cast<unsigned>(ycol) < 32u);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               float2 zz = make_float2(v[2 * j], v[2 * j + 1]);
@@ -620,8 +631,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 e0 = col < ncols ? e0 : 0.f;
                 e1 = col + 1 < ncols ? e1 : 0.f;
               }
-              sacc = __fadd2_rn(sacc, make_float2(e0, e1));
-              uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
+              float2 es = make_float2(e0, e1);
+              if (tgt) {
+                es.x = 2 * j == ycol ? 0.f : e0;
+                es.y = 2 * j + 1 == ycol ? 0.f : e1;
+              }
+              sacc = __fadd2_rn(sacc, es);
+              const float2 ds =
+                  __fadd2_rn(make_float2(v[2 * j], v[2 * j + 1]), make_float2(-cs, -cs));
+              uacc = __ffma2_rn(es, ds, uacc);
               p[j] = pack_bf16x2(e0, e1);
             }
 #pragma unroll

@@ -86,7 +86,8 @@ struct GemmArgs {
   int32_t aux_slots;       // slots in the auxiliary buffer
   // kLogits epilogue
   const int32_t* targets;  // [M] token targets (flattened [K, N])
-  float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile
+  float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile; kLogits /
+                           //   kLogitsHeads leave the target's own term out of the sum
   float* zy;               // [M]: logit of the target
   int32_t V;
   uint32_t* flags;         // device flag word
@@ -164,6 +165,8 @@ struct RowArgs {
   float* zy;            // [M]
   float* edz;           // [M]: E_p[s] - s_y per kept token (0 if masked), for the
                         //      RMSNorm backward's row sum
+  float* nll;           // [M]: lse - z_y of a row whose target is in range (the
+                        //      gradient's p_y - 1 = expm1(-nll) keeps its precision)
   float2* stats;        // [n_tiles_v, M]
   double* part_sum;     // [K, part_blocks]
   int32_t* part_cnt;    // [K, part_blocks]

@@ -221,6 +221,15 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     const int64_t row = static_cast<int64_t>(k) * a.N + n;
     float mx = -INFINITY, s = 0.f, us = 0.f;
     int best_tile = 0;
+    // E_p[s] - s_y = sum_t e^{m_t - M} (u_t + (c_t - s_y) s_t) / sum_t e^{m_t - M} s_t,
+    // u_t = sum over the tile of exp(z - m_t) (s - c_t), c_t = m_t / tau (as in
+    // the logits epilogue)
+    float ys = 0.f, tau = 1.f;
+    if constexpr (!kExit) {
+      const int y0 = a.targets ? a.targets[row] : a.ignore_index;
+      if (token_kept(a, row, y0)) ys = kHeads ? a.sy[row] : a.zy[row];
+      if (kHeads && a.tau) tau = a.tau[k];
+    }
     for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
       float2 st[8];
       float uu[8];
@@ -243,22 +252,36 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       for (int u = 0; u < 8; ++u) {
         const float f = expf(st[u].x - cm);
         s += st[u].y * f;
-        if constexpr (!kExit) us += uu[u] * f;
+        if constexpr (!kExit) {
+          if (t0 + u < a.n_tiles_v) {         // padding tiles have m = -inf
+            const float c = tau != 0.f ? st[u].x / tau : 0.f;
+            us += (uu[u] + (c - ys) * st[u].y) * f;
+          }
+        }
       }
       mx = cm;
-    }
-    const float l = mx + logf(s);
-    if constexpr (kExit) {
-      if (a.top1 && in_bounds(best_tile < a.n_tiles_v, a.flags))
-        a.top1[row] = a.argmax[static_cast<int64_t>(best_tile) * M + row];
-      if (a.top1_logprob) a.top1_logprob[row] = mx - l;
-    } else {
-      a.lse[row] = l;
     }
     const int y = a.targets ? a.targets[row] : a.ignore_index;
     bad = !(y >= 0 && y < a.V) && y != a.ignore_index;
     const bool kept = token_kept(a, row, y);
-    const float loss = kept ? l - a.zy[row] : 0.f;
+    float l = mx + logf(s), nll = 0.f;
+    if constexpr (kExit) {
+      if (a.top1 && in_bounds(best_tile < a.n_tiles_v, a.flags))
+        a.top1[row] = a.argmax[static_cast<int64_t>(best_tile) * M + row];
+      if (a.top1_logprob) a.top1_logprob[row] = mx - l;
+      nll = l - a.zy[row];
+    } else {
+      if (y >= 0 && y < a.V) {
+        // the tile sums leave the target's term out: lse - z_y without
+        // cancellation (mx >= z_y, equal when the target holds the maximum)
+        const float zt = a.zy[row];
+        nll = zt >= mx ? log1pf(s * expf(mx - zt)) : (mx - zt) + logf(s + expf(zt - mx));
+        l = zt + nll;
+        a.nll[row] = nll;
+      }
+      a.lse[row] = l;
+    }
+    const float loss = kept ? nll : 0.f;
     if (a.loss_tok) a.loss_tok[row] = loss;
     lsum = loss;
     cnt = kept ? 1 : 0;
@@ -266,7 +289,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       // E_p[s] - s_y (s: the logits before temperature and bias; s = z
       // without them): the temperature's gradient term and, scaled, the
       // RMSNorm backward's row sum
-      const float e = kept ? us / s - (kHeads ? a.sy[row] : a.zy[row]) : 0.f;
+      const float e = kept ? us * expf(mx - l) : 0.f;   // the sums are relative to mx
       a.edz[row] = e;
       if constexpr (kHeads) tsum = e;
     }
@@ -336,7 +359,8 @@ __global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
 // ---- dL/dz in place: G = tau (softmax - onehot) / Nvalid --------------------
 // The buffer holds p~ = bf16(exp(z - m_t)) for the column tile t of each
 // entry, so softmax = p~ * exp(m_t - lse).  The target entry is recomputed
-// from the fp32 target logit so that p_y - 1 keeps its relative precision.
+// as expm1(-(lse - z_y)), from the lse - z_y that the log-sum-exp pass forms
+// without cancellation, so that p_y - 1 keeps its relative precision.
 
 // One row per CTA: contiguous 16-byte vectors across the row (the fastest
 // form; used when no bias gradient is needed).
@@ -358,7 +382,7 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   const float l = a.lse[row];
   for (int t = threadIdx.x; t < a.n_tiles_v; t += 256)
     ctile[t] = expf(a.stats[static_cast<int64_t>(t) * M + row].x - l) * w;
-  const float gy = (expf(a.zy[row] - l) - 1.0f) * w;
+  const float gy = expm1f(-a.nll[row]) * w;    // p_y - 1 at full relative precision
   __syncthreads();
   for (int v = threadIdx.x; v < nvec; v += 256) {
     const int v0 = v * 8;
@@ -410,7 +434,7 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
       cfac[r][tt] = (wr != 0.f && t < a.n_tiles_v)
                         ? expf(a.stats[static_cast<int64_t>(t) * M + i].x - l) * wr : 0.f;
     }
-    sgy[r] = kept ? (expf(a.zy[i] - l) - 1.0f) * wr : 0.f;
+    sgy[r] = kept ? expm1f(-a.nll[i]) * wr : 0.f;
     sy[r] = kept ? y : -1;
   }
   __syncthreads();

@@ -54,7 +54,8 @@ struct Layout {
   int part_blocks = 0;
   int dg_chunks = 0;
   int db_chunks = 0;
-  size_t flags = 0, r = 0, lse = 0, zy = 0, edz = 0, part_sum = 0, part_cnt = 0, inv_nvalid = 0;
+  size_t flags = 0, r = 0, lse = 0, zy = 0, edz = 0, nll = 0, part_sum = 0, part_cnt = 0;
+  size_t inv_nvalid = 0;
   size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
   int aux_slots = 0;
@@ -95,6 +96,7 @@ Layout make_layout(const solo_dims_t& d) {
   L.lse = take(M * 4);
   L.zy = take(M * 4);
   L.edz = take(M * 4);
+  L.nll = take(M * 4);
   L.part_sum = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
   L.part_cnt = take(static_cast<size_t>(d.K) * L.part_blocks * 4);
   L.inv_nvalid = take(SOLO_MAX_MODULES * 4);
@@ -296,6 +298,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.lse = reinterpret_cast<float*>(ws + L.lse);
   ra.zy = reinterpret_cast<float*>(ws + L.zy);
   ra.edz = reinterpret_cast<float*>(ws + L.edz);
+  ra.nll = reinterpret_cast<float*>(ws + L.nll);
   ra.stats = reinterpret_cast<float2*>(ws + L.stats);
   ra.part_sum = reinterpret_cast<double*>(ws + L.part_sum);
   ra.part_cnt = reinterpret_cast<int32_t*>(ws + L.part_cnt);
