@@ -585,13 +585,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                      fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
         }
         const float mlog = mx * kLog2e;
-        // the sum of exp(z - m) in two lanes of a packed pair (even and odd columns)
+        // the sums of exp(z - m) and of exp(z - m) s, each in the two lanes of a
+        // packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
-        // sum of exp(z - m) (s - c), likewise, with c = m / tau: near the tile
-        // maximum s - c is small, so a confident row's E_p[s] - s_y keeps its
-        // relative precision (the log-sum-exp pass adds (c - s_y) times the
-        // sum of exp back per tile, with the same c)
-        const float cs = tau != 0.f ? mx / tau : 0.f;
         float2 uacc = make_float2(0.f, 0.f);
         for (int cp = 0; cp < kBN / 64; ++cp) {
           if (cp * 64 >= ncols) break;
@@ -611,19 +607,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             }
             uint32_t p[16];
             const bool ragged = c * 32 + 32 > ncols;      // warp-uniform
-            // The target's own term is left out of the tile's sums (the
-            // stored exponential keeps it): the log-sum-exp pass then forms
-            // lse - z_y = log1p(sum over v != y of exp(z_v - z_y)), and 1 - p_y
-            // and E_p[s] - s_y of a confident row do not cancel.
+            float z[32];
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) {
+              float2 zz = make_float2(v[j], v[j + 1]);
+              if constexpr (kHeads)
+                zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[j], bb[j + 1]));
+              z[j] = zz.x;
+              z[j + 1] = zz.y;
+            }
+            // The target's own term is left out of the tile's sums and of the
+            // stored exponentials (the gradient pass writes the target entry
+            // itself): the log-sum-exp pass forms lse - z_y = log1p(sum over
+            // v != y of exp(z_v - z_y)), so that 1 - p_y and E_p[s] - s_y of a
+            // confident row do not cancel.
             const int ycol = has_y ? yrel - c * 32 : -1;
-            const bool tgt = __any_sync(0xffffffffu, static_cast<unsigned>(ycol) < 32u);
+            if (__any_sync(0xffffffffu, static_cast<unsigned>(ycol) < 32u)) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) z[j] = j == ycol ? -INFINITY : z[j];
+            }
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              float2 zz = make_float2(v[2 * j], v[2 * j + 1]);
-              if constexpr (kHeads)
-                zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[2 * j], bb[2 * j + 1]));
-              const float2 a =
-                  __ffma2_rn(zz, make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
+              const float2 a = __ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]),
+                                          make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
               float e0 = ex2_approx(a.x);
               float e1 = ex2_approx(a.y);
               if (ragged) {
@@ -631,15 +637,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 e0 = col < ncols ? e0 : 0.f;
                 e1 = col + 1 < ncols ? e1 : 0.f;
               }
-              float2 es = make_float2(e0, e1);
-              if (tgt) {
-                es.x = 2 * j == ycol ? 0.f : e0;
-                es.y = 2 * j + 1 == ycol ? 0.f : e1;
-              }
-              sacc = __fadd2_rn(sacc, es);
-              const float2 ds =
-                  __fadd2_rn(make_float2(v[2 * j], v[2 * j + 1]), make_float2(-cs, -cs));
-              uacc = __ffma2_rn(es, ds, uacc);
+              sacc = __fadd2_rn(sacc, make_float2(e0, e1));
+              uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
               p[j] = pack_bf16x2(e0, e1);
             }
 #pragma unroll

@@ -221,14 +221,12 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     const int64_t row = static_cast<int64_t>(k) * a.N + n;
     float mx = -INFINITY, s = 0.f, us = 0.f;
     int best_tile = 0;
-    // E_p[s] - s_y = sum_t e^{m_t - M} (u_t + (c_t - s_y) s_t) / sum_t e^{m_t - M} s_t,
-    // u_t = sum over the tile of exp(z - m_t) (s - c_t), c_t = m_t / tau (as in
-    // the logits epilogue)
-    float ys = 0.f, tau = 1.f;
+    // E_p[s] - s_y = e^{M - lse} sum_t e^{m_t - M} (u_t - s_y s_t), with the
+    // target's term left out of the tile sums s_t and u_t = sum of exp(z - m_t) s
+    float ys = 0.f;
     if constexpr (!kExit) {
       const int y0 = a.targets ? a.targets[row] : a.ignore_index;
       if (token_kept(a, row, y0)) ys = kHeads ? a.sy[row] : a.zy[row];
-      if (kHeads && a.tau) tau = a.tau[k];
     }
     for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
       float2 st[8];
@@ -253,10 +251,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
         const float f = expf(st[u].x - cm);
         s += st[u].y * f;
         if constexpr (!kExit) {
-          if (t0 + u < a.n_tiles_v) {         // padding tiles have m = -inf
-            const float c = tau != 0.f ? st[u].x / tau : 0.f;
-            us += (uu[u] + (c - ys) * st[u].y) * f;
-          }
+          us += fmaf(-ys, st[u].y, uu[u]) * f;   // padding tiles add 0: f = 0, s_t = u_t = 0
         }
       }
       mx = cm;
