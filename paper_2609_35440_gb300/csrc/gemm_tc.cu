@@ -230,7 +230,8 @@ __device__ __forceinline__ void norm_bwd_chunk(const GemmArgs& g, const float (&
 }
 
 // The dgamma partial row of the 32-row block starting at row_base (a multiple
-// of 32), for columns from col0; null when the block holds no final-module row.
+// of 32), for columns from col0.  Callers ask only for blocks holding a row of
+// the final module; a checked build tests that and returns null otherwise.
 __device__ __forceinline__ float* dg_block(const GemmArgs& g, int64_t row_base, int col0) {
   const int64_t rb = (row_base >> 5) - (g.dg_row0 >> 5);
   if (g.dg_part == nullptr || !in_bounds(rb >= 0 && rb < g.dg_blocks, g.flags)) return nullptr;

@@ -96,7 +96,8 @@ struct GemmArgs {
   const float* tau;        // [K] or null (1)
   const float* bias;       // [K, V] or null (0)
   int64_t tokens_per_module;
-  float* usum;             // [n_blocks, M]: sum over the tile of exp(z - m) * s
+  float* usum;             // [n_blocks, M]: sum over the tile of exp(z - m) * s (the
+                           //   target's term left out, like the sum in stats)
   float* sy;               // [M]: s at the target (before temperature and bias)
   // kDxhat with the RMSNorm backward fused into the epilogue (norm_fused = 1):
   // whole tiles write dH = r gamma dxhat - (r^3 / d) h S in bf16 and the final
