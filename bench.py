@@ -92,6 +92,28 @@ def load_peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
+SUSTAINED_AFTER_S = 1.0   # timed regions at least this long run under the power cap
+
+
+def tensor_peak(peaks, src: str, timed_s: float):
+    """The bf16 peak that matches how the kernels were timed: the burst figure
+    (torch.matmul best of 10) for a timed region shorter than a second, the
+    sustained one (seconds back to back under the power cap) otherwise."""
+    if timed_s < SUSTAINED_AFTER_S:
+        key, why = "bf16_tflops", f"timed region {timed_s:.2f} s < {SUSTAINED_AFTER_S:.0f} s"
+    else:
+        key, why = "bf16_tflops_sustained", f"timed region {timed_s:.2f} s >= " \
+                                            f"{SUSTAINED_AFTER_S:.0f} s"
+    return float(peaks.get(key, FALLBACK_PEAKS[key])), f"{src} {key} ({why})"
+
+
+def kept_counts(wl, targets) -> list:
+    """Kept tokens per module: targets in [0, V) (ignore_index and anything out
+    of range are masked, as the library treats them)."""
+    t = np.asarray(targets)
+    return [int(np.sum((t[k] >= 0) & (t[k] < wl.V))) for k in range(wl.K)]
+
+
 def strip_comments(src: str) -> str:
     """C++ source without comments, every run of whitespace made one space, so
     that neither comments nor layout count as a change of the code (string
@@ -221,7 +243,8 @@ def replica_workload(wl, rank: int):
 E2E_METHOD = ("every step: its hidden states and targets copied from pinned host memory "
               "into one of two device buffers on a copy stream (overlapping the previous "
               "step's compute), the call, and its losses copied back; all inside the timed "
-              "region")
+              "region.  Returned to the host: loss_tok and loss_mean only; dH, dW and dgamma "
+              "stay on the device for the caller's backward pass")
 
 def pipelined_e2e(torch, dev, stream, h_host, t_host, hidden, targets, compute, read_back,
                   steps, warm=2):
@@ -488,9 +511,10 @@ def run_ours(args, wl):
     dom = max(gemm_stage_flops, key=lambda s: stage_ms[names.index(s)])
     dom_ms = stage_ms[names.index(dom)]
     achieved = gemm_stage_flops[dom] / (dom_ms / 1e3) / 1e12
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
     traffic = committed_traffic(wl) if dom == "logits" else None
     algo = costmodel.call_flops(wl.K, wl.N, wl.d, wl.V)
+    kept = costmodel.kept_call_flops(kept_counts(wl, inp.targets), wl.d, wl.V)
     step_s = ms / 1e3 / args.steps
     cpu = None
     if not args.no_cpu:
@@ -505,7 +529,12 @@ def run_ours(args, wl):
                    "global_batch_tokens": world * wl.M, "parallelism": f"replicas{world}",
                    "l2": l2_note(wl, True)},
         "algo_tflops": algo / step_s / 1e12,
+        # the whole call's algorithmic rate against the same peak as the roofline
         "algo_frac_of_peak": algo / step_s / 1e12 / peak,
+        # the paper's work on kept tokens only (masked tokens still run through
+        # every product; the mean loss counts kept tokens)
+        "kept_algo_tflops": kept / step_s / 1e12,
+        "kept_algo_frac_of_peak": kept / step_s / 1e12 / peak,
         # the tensor cores execute exactly the algorithmic (2K+1) 2NVd: no logits
         # are recomputed (the forward stores its exponentials)
         "executed_tflops": algo / step_s / 1e12,
@@ -513,8 +542,7 @@ def run_ours(args, wl):
         "roofline": {"bound": "tensor", "kernel": f"{dom} GEMM (tcgen05)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside "
-                                    f"back-to-back steps)"},
+                     "peak_source": peak_name},
         "cpu_baseline": cpu,
         "e2e": e2e,
         "clocks": clk.summary(),
@@ -598,7 +626,7 @@ def run_exit_bench(args, wl):
     ems = pipelined_e2e(torch, dev, stream, h_host, t_host, hidden, targets, compute, read_back,
                         steps_e2e)
     peaks, peak_src = load_peaks()
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
     G = costmodel.gemm_flops(wl.M, wl.V, wl.d)
     achieved = G / (stage_ms[1] / 1e3) / 1e12
     cpu = None
@@ -629,12 +657,14 @@ def run_exit_bench(args, wl):
         "roofline": {"bound": "tensor", "kernel": "exit logits GEMM (tcgen05)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None,
-                     "peak_source": f"{peak_src} bf16_tflops_sustained"},
+                     "peak_source": peak_name},
         "cpu_baseline": cpu,
         "e2e": {"value": job_throughput(wl.M, steps_e2e, 1, ems), "unit": "tokens/s",
                 "h2d_bytes_per_step": sum(h.numel() * 2 for h in h_host) + t_host.numel() * 4,
                 "d2h_bytes_per_step": lt_host.numel() * 4 + top_host.numel() * 4,
-                "method": E2E_METHOD.replace("its losses", "its losses and top-1")},
+                "method": E2E_METHOD.split("  Returned")[0].replace(
+                    "its losses", "its losses and top-1") +
+                          "  Returned to the host: loss_tok and top1"},
         "clocks": clk.summary(),
         "gpu_launches": launches,       # the library's own count over the timed calls
         "device_flags": flags,
@@ -685,7 +715,7 @@ def run_private_bench(args, wl):
     clk.__exit__(None, None, None)
     ms = t0.elapsed_time(t1)
     peaks, peak_src = load_peaks()
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
     algo = 3 * K * costmodel.gemm_flops(N, V, d)      # per module: logits, dX, dW_k
     tflops = algo / (ms / args.steps / 1e3) / 1e12
     line = {"metric": PRIVATE_METRIC, "value": job_throughput(wl.M, args.steps, 1, ms),
@@ -696,7 +726,7 @@ def run_private_bench(args, wl):
                        "parallelism": "replicas1", "l2": l2_note(wl, True)},
             "algo_tflops": tflops,
             "algo_frac_of_peak": tflops / peak,
-            "peak_source": f"{peak_src} bf16_tflops_sustained",
+            "peak_source": peak_name,
             "clocks": clk.summary(), "gpu_launches": launches,
             "device_flags": sr.solo_readout_get_flags(ws, stream)}
     print(json.dumps(line), flush=True)

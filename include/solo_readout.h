@@ -50,7 +50,8 @@ typedef int32_t solo_status_t;
 enum {
   SOLO_OK = 0,
   SOLO_ERR_INVALID_ARG = -1,         /* NULL required pointer, K/N/d/V out of range */
-  SOLO_ERR_UNSUPPORTED_SHAPE = -2,   /* d not a multiple of 8 */
+  SOLO_ERR_UNSUPPORTED_SHAPE = -2,   /* d not a multiple of 8, V above 2^23, or K*N
+                                        beyond 32-bit tile coordinates */
   SOLO_ERR_WORKSPACE_TOO_SMALL = -3, /* workspace_bytes below the query result */
   SOLO_ERR_CUDA = -4,                /* a CUDA runtime call failed */
   SOLO_ERR_NOT_SM103 = -5,           /* current device is not compute capability 10.3 */
@@ -94,7 +95,7 @@ typedef struct {
   int32_t K;            /* modules, 1 .. SOLO_MAX_MODULES                    */
   int64_t N;            /* tokens per module, >= 1                           */
   int32_t d;            /* width, >= 8 and a multiple of 8                   */
-  int32_t V;            /* vocabulary size, >= 1                             */
+  int32_t V;            /* vocabulary size, 1 .. 2^23                        */
   float eps;            /* RMSNorm epsilon, inside the square root (>= 0)    */
   int32_t ignore_index; /* target value of a masked token (e.g. -100)        */
 } solo_dims_t;
@@ -103,9 +104,9 @@ typedef struct {
  * Bytes of device workspace one call with these dims needs (host-only; no
  * CUDA call).  The workspace holds the normalised inputs, the bf16
  * exponentials/gradient of the logits ([K*N, V]), per-token statistics,
- * fp32 partial tiles of the backward products and the flag word.  Returns
- * SOLO_ERR_INVALID_ARG for NULL pointers or dims out of range,
- * SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0.
+ * at most 32 MiB of fp32 partial tiles of the backward products and the flag
+ * word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims out of range,
+ * SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0 or V > 2^23.
  */
 solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
 
@@ -395,12 +396,17 @@ uint64_t solo_readout_kernel_launches(void);
  *  - Problems whose solo_readout_workspace_bytes exceeds
  *    SOLO_STATIC_SCRATCH_BYTES are rejected with
  *    SOLO_ERR_EXCEEDS_STATIC_SCRATCH before anything is enqueued (roughly
- *    K*N*(2.0625*V + 6*d + 24) bytes plus up to 32 MiB of partial tiles of the
+ *    K*N*(2.0625*V + 2*d + 24) bytes plus up to 32 MiB of partial tiles of the
  *    backward products must fit; e.g. K=2, N=256, d=128, V=4096 uses about
- *    8.5 MiB).
+ *    8.3 MiB).
  *  - The first call on a device looks up the device address of the scratch
  *    array for that device (the array's name in host code is not a device
- *    address).  Make that first call before any stream capture.
+ *    address) and keeps it for the rest of the process.  Make that first call
+ *    before any stream capture.  A cudaDeviceReset destroys the device's
+ *    context and the array with it, so the kept address (like the kernel
+ *    attributes every entry point sets on its first call on a device) is no
+ *    longer valid: after a reset, do not call this library on that device
+ *    again in the same process.
  *  - Every call on a device shares the one array, and it keeps the previous
  *    call's contents; the call clears what must start at zero itself.  Calls
  *    whose execution overlaps on the GPU (other streams, other host

@@ -52,6 +52,15 @@ def call_flops(K: int, N: int, d: int, V: int) -> float:
     return (2 * K + 1) * 2.0 * N * V * d
 
 
+def kept_call_flops(n_kept, d: int, V: int) -> float:
+    """Algorithmic tensor FLOPs spent on kept tokens only: 2r = 4Vd per kept
+    token of an auxiliary module and 3r = 6Vd per kept token of the final one
+    (``n_kept``: kept-token counts of the K modules, final module last).  The
+    call itself still runs masked tokens through every product."""
+    n = [int(x) for x in n_kept]
+    return 4.0 * V * d * sum(n[:-1]) + 6.0 * V * d * n[-1]
+
+
 def gemm_flops(M: int, N: int, Kdim: int) -> float:
     return 2.0 * M * N * Kdim
 

@@ -708,10 +708,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            if (part == 0) {
+            if (part == 0 && !args.aux_part0) {
               tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
-            } else {    // a later reduction range of a cut tile: its auxiliary slot
-              const int slot = (t - args.full_tiles) * (args.split - 1) + part - 1;
+            } else {    // a reduction range of a cut tile: its auxiliary slot
+              const int cut = t - args.full_tiles;
+              const int slot = args.aux_part0 ? cut * args.split + part
+                                              : cut * (args.split - 1) + part - 1;
               if (in_bounds(slot >= 0 && slot < args.aux_slots, args.flags))
                 tma_store_2d(&tmX, ebuf + buf * kEpiBufBytes, c * 32,
                              slot * kPairRows + static_cast<int>(rank) * kBM + 32 * q);
@@ -769,7 +771,7 @@ void plan_units(GemmArgs& g, int sms, bool allow_split) {
   const int rem = g.num_tiles % pairs;
   if (!allow_split || rem == 0) return;
   int s = std::min({pairs / rem, kMaxSplit, g.k_blocks});
-  while (s > 1 && rem * (s - 1) > kMaxAuxSlots) --s;
+  while (s > 1 && rem * (g.aux_part0 ? s : s - 1) > std::min(g.aux_slots, kMaxAuxSlots)) --s;
   if (s < 2) return;
   g.full_tiles = g.num_tiles - rem;
   g.split = s;
@@ -809,15 +811,18 @@ __global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, floa
   }
 }
 
-// kDxhat with norm_fused: the RMSNorm backward of the cut tiles, from their
-// fp32 dX̂ summed by split_fixup_kernel.  Grid (cut tiles, 8 blocks of 32
+// kDxhat with norm_fused: the RMSNorm backward of the cut tiles, from the sum
+// of their fp32 parts in the auxiliary buffer (part 0 first, then 1, 2, ...:
+// the order split_fixup_kernel adds them in).  Grid (cut tiles, 8 blocks of 32
 // rows); warp w handles the tile's columns [32 w, 32 w + 32), lane i row i.
-__global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, const float* dxhat) {
-  const int t = g.full_tiles + static_cast<int>(blockIdx.x);
+__global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, const float* aux) {
+  const int cut = static_cast<int>(blockIdx.x);
+  const int t = g.full_tiles + cut;
   int mb, nb;
   tile_coords(t, g, mb, nb);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int lr = blockIdx.y * 32 + lane;                    // row within the tile
   const int64_t row_base = static_cast<int64_t>(mb) * kPairRows + blockIdx.y * 32;
   const int64_t row = row_base + lane;
   const int col0 = nb * kBN + warp * 32;
@@ -826,14 +831,31 @@ __global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, c
   const NormRow nr = norm_row(g, row);
   float v[32];
 #pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (nr.ok && 4 * q < cols)
-      x = *reinterpret_cast<const float4*>(dxhat + row * g.N + col0 + 4 * q);
-    v[4 * q] = x.x;
-    v[4 * q + 1] = x.y;
-    v[4 * q + 2] = x.z;
-    v[4 * q + 3] = x.w;
+  for (int j = 0; j < 32; ++j) v[j] = 0.f;
+  if (nr.ok) {
+    for (int p = 0; p < g.split; ++p) {
+      const int slot = cut * g.split + p;
+      if (!in_bounds(slot < g.aux_slots, g.flags)) continue;
+      const float4* src = reinterpret_cast<const float4*>(
+          aux + (static_cast<int64_t>(slot) * kPairRows + lr) * kBN + warp * 32);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (4 * q < cols) {
+          const float4 x = src[q];
+          if (p == 0) {
+            v[4 * q] = x.x;
+            v[4 * q + 1] = x.y;
+            v[4 * q + 2] = x.z;
+            v[4 * q + 3] = x.w;
+          } else {
+            v[4 * q] += x.x;
+            v[4 * q + 1] += x.y;
+            v[4 * q + 2] += x.z;
+            v[4 * q + 3] += x.w;
+          }
+        }
+      }
+    }
   }
   const bool dg_warp = __any_sync(0xffffffffu, nr.dg);
   norm_bwd_chunk(g, v, col0, cols, nr, dg_warp, dg_warp ? dg_block(g, row_base, col0) : nullptr);
@@ -841,10 +863,10 @@ __global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, c
 
 }  // namespace
 
-cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* dxhat, cudaStream_t stream) {
+cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* aux, cudaStream_t stream) {
   const int cut = g.num_tiles - g.full_tiles;
-  if (!g.norm_fused || g.split < 2 || cut <= 0) return cudaSuccess;
-  cut_tiles_norm_kernel<<<dim3(cut, kPairRows / 32), 256, 0, stream>>>(g, dxhat);
+  if (!g.norm_fused || !g.aux_part0 || g.split < 2 || cut <= 0) return cudaSuccess;
+  cut_tiles_norm_kernel<<<dim3(cut, kPairRows / 32), 256, 0, stream>>>(g, aux);
   return launched();
 }
 

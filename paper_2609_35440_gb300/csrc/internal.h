@@ -79,11 +79,16 @@ struct GemmArgs {
   // into `split` contiguous reduction ranges (fills the last partial wave of
   // CTA pairs).  Part 0 of a cut tile is stored to the output, parts 1.. to
   // the auxiliary buffer (slot (tile - full_tiles) * (split - 1) + part - 1,
-  // 256 x 256 fp32 each) and added by launch_split_fixup in a fixed order.
+  // 256 x 256 fp32 each) and added by launch_split_fixup in a fixed order
+  // (with aux_part0, every part goes to the auxiliary buffer).
   int32_t full_tiles;
   int32_t split;
   int32_t num_units;
   int32_t aux_slots;       // slots in the auxiliary buffer
+  int32_t aux_part0;       // 1: part 0 of a cut tile goes to the auxiliary buffer as
+                           //   well (slot (tile - full_tiles) * split + part), and the
+                           //   output is never written for cut tiles (kDxhat with the
+                           //   fused RMSNorm backward: cut_tiles_norm sums the parts)
   // kLogits epilogue
   const int32_t* targets;  // [M] token targets (flattened [K, N])
   float2* stats;           // [n_blocks, M]: (max, sum exp(z - max)) per tile; kLogits /
@@ -101,7 +106,7 @@ struct GemmArgs {
   float* sy;               // [M]: s at the target (before temperature and bias)
   // kDxhat with the RMSNorm backward fused into the epilogue (norm_fused = 1):
   // whole tiles write dH = r gamma dxhat - (r^3 / d) h S in bf16 and the final
-  // module's dgamma partial sums; cut tiles store fp32 dXhat as without it.
+  // module's dgamma partial sums; cut tiles store their fp32 parts (aux_part0).
   int32_t norm_fused;
   int32_t modules;                       // K
   const uint16_t* hidden[kMaxModules];   // [N, d] bf16 per module
@@ -120,18 +125,19 @@ cudaError_t gemm_prepare(int device);  // sets the dynamic shared memory limit o
 
 constexpr int kMaxSplit = 8;        // reduction ranges per cut tile
 constexpr int kMaxAuxSlots = 127;   // 256 x 256 fp32 partial tiles (32 MB)
-// Auxiliary slots a product of `tiles` tiles and `k_blocks` reduction blocks
-// may need (a part keeps at least one reduction block).
-inline int split_aux_slots(int64_t tiles, int64_t k_blocks) {
-  const int64_t parts = k_blocks < kMaxSplit ? k_blocks : kMaxSplit;
-  const int64_t s = tiles * (parts - 1);
-  return static_cast<int>(s < kMaxAuxSlots ? s : kMaxAuxSlots);
-}
 // Sets full_tiles / split / num_units: whole tiles fill complete waves of
 // min(sms / 2, kMaxAuxSlots + 1) pairs; the remainder is cut so the last wave
-// has as many units as pairs (each part keeps >= 1 reduction block).
-// allow_split = false keeps every tile whole.
+// has as many units as pairs (each part keeps >= 1 reduction block) and its
+// parts fit in g.aux_slots (g.aux_part0: every part takes a slot; otherwise
+// part 0 goes to the output).  allow_split = false keeps every tile whole.
 void plan_units(GemmArgs& g, int sms, bool allow_split);
+// Slots a product needs at most: `tiles` tiles of `k_blocks` reduction
+// blocks, with (part0 = true) or without part 0 in the auxiliary buffer.
+inline int split_aux_slots(int64_t tiles, int64_t k_blocks, bool part0) {
+  const int64_t parts = k_blocks < kMaxSplit ? k_blocks : kMaxSplit;
+  const int64_t s = tiles * (part0 ? parts : parts - 1);
+  return static_cast<int>(s < kMaxAuxSlots ? s : kMaxAuxSlots);
+}
 // Launches min(units, sms / 2) CTA pairs.  x: tensor map of the auxiliary
 // buffer (fp32 [slots * 256, 256], 32 x 32 boxes) for the cut tiles' parts.
 cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& b,
@@ -140,9 +146,10 @@ cudaError_t launch_gemm(GemmMode mode, const CUtensorMap& a, const CUtensorMap& 
 // out (fp32, row stride ld) += the auxiliary parts of every cut tile.
 cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const float* aux,
                                cudaStream_t stream);
-// kDxhat with norm_fused, after launch_split_fixup: the RMSNorm backward (dH,
-// dgamma partials) of the cut tiles, from their summed fp32 dXhat.
-cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* dxhat, cudaStream_t stream);
+// kDxhat with norm_fused (and aux_part0): the RMSNorm backward (dH, dgamma
+// partials) of the cut tiles, from the sum of their parts in the auxiliary
+// buffer, added in part order.
+cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* aux, cudaStream_t stream);
 
 // ---- row kernels ---------------------------------------------------------------
 

@@ -10,7 +10,7 @@
 //   dxhat        tensor-core G W with the RMSNorm backward in its epilogue:
 //                bf16 dH and the final module's dgamma partial sums [K*N, d]
 //   norm_bwd     the same for the tiles whose last wave was cut along V
-//                (their fp32 dXhat summed first)
+//                (their fp32 parts summed first, from the partial-tile slots)
 //   dW           tensor-core G^T xhat over the final module       [V, d]
 //   dgamma       fixed-order sum of the partials                  [d]
 #include <cudaTypedefs.h>
@@ -40,6 +40,9 @@ namespace {
 using namespace solo;
 
 constexpr size_t kAlign = 1024;
+// Largest vocabulary: the gradient pass keeps one float per 256-column tile of
+// a row in shared memory (128 KB at this size).
+constexpr int32_t kMaxVocab = 1 << 23;
 // Tile raster (in 256-row pair blocks) per product, from a sweep on GB300.
 constexpr int kGroupLogits = 16;
 constexpr int kGroupDxhat = 4;
@@ -56,7 +59,7 @@ struct Layout {
   int db_chunks = 0;
   size_t flags = 0, r = 0, lse = 0, zy = 0, edz = 0, nll = 0, part_sum = 0, part_cnt = 0;
   size_t inv_nvalid = 0;
-  size_t stats = 0, xhat = 0, P = 0, dxhat = 0, dgp = 0;
+  size_t stats = 0, xhat = 0, P = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
   int aux_slots = 0;
 };
@@ -70,7 +73,11 @@ solo_status_t check_dims(const solo_dims_t* d) {
   // row and column coordinates of the tensor-core operands are 32-bit
   const int64_t M = static_cast<int64_t>(d->K) * d->N;
   if (M > (int64_t{1} << 31) - 1 - kBM) return SOLO_ERR_UNSUPPORTED_SHAPE;
-  if (d->V > (1 << 30) || d->d > (1 << 20)) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  if (d->V > kMaxVocab || d->d > (1 << 20)) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  // tile counts of the products are 32-bit
+  const int64_t row_blocks = (M + 2 * kBM - 1) / (2 * kBM);
+  const int64_t col_blocks = (static_cast<int64_t>(d->V) + kBN - 1) / kBN;
+  if (row_blocks * col_blocks > (int64_t{1} << 31) - 1) return SOLO_ERR_UNSUPPORTED_SHAPE;
   return SOLO_OK;
 }
 
@@ -103,19 +110,19 @@ Layout make_layout(const solo_dims_t& d) {
   L.stats = take(static_cast<size_t>(L.n_tiles_v) * M * 8);
   L.xhat = take(M * d.d * 2);
   L.P = take(M * static_cast<size_t>(L.ldp) * 2);
-  L.dxhat = take(M * d.d * 4);
   L.dgp = take(static_cast<size_t>(L.dg_chunks) * d.d * 4);
   // heads' temperature and bias gradients
   L.usum = take(static_cast<size_t>(L.n_tiles_v) * M * 4);
   L.sy = take(M * 4);
   L.part_tau = take(static_cast<size_t>(d.K) * L.part_blocks * 8);
   L.db_part = take(static_cast<size_t>(d.K) * L.db_chunks * L.ldp * 4);
-  // partial tiles of the dX̂ and dW products' last wave (one at a time)
+  // partial tiles of the dX̂ and dW products' last wave (one product at a
+  // time; every part of a cut dX̂ tile, parts 1.. of a cut dW tile)
   const int64_t nb = (d.d + kBN - 1) / kBN;
   const int64_t tiles_dx = (L.M + 2 * kBM - 1) / (2 * kBM) * nb;
   const int64_t tiles_dw = (d.V + 2 * kBM - 1) / (2 * kBM) * nb;
-  L.aux_slots = std::max(split_aux_slots(tiles_dx, (d.V + kBK - 1) / kBK),
-                         split_aux_slots(tiles_dw, (d.N + kBK - 1) / kBK));
+  L.aux_slots = std::max(split_aux_slots(tiles_dx, (d.V + kBK - 1) / kBK, true),
+                         split_aux_slots(tiles_dw, (d.N + kBK - 1) / kBK, false));
   L.aux = take(static_cast<size_t>(std::max(L.aux_slots, 1)) * 2 * kBM * kBN * 4);
   L.total = off;
   return L;
@@ -307,7 +314,6 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.loss_tok = loss_tok;
   ra.loss_mean = loss_mean;
   ra.P = reinterpret_cast<uint16_t*>(ws + L.P);
-  float* dxhat = reinterpret_cast<float*>(ws + L.dxhat);
   ra.dgamma_part = reinterpret_cast<float*>(ws + L.dgp);
   ra.dg_chunks = L.dg_chunks;
   ra.dgamma = dgamma;
@@ -326,7 +332,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   const uint64_t V = static_cast<uint64_t>(D.V);
   const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
-  CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mDX, mG_mn, mX_mn, mDW, mAux;
+  CUtensorMap mX_k, mW_k, mP_st, mG_k, mW_mn, mG_mn, mX_mn, mDW, mAux;
   float* aux = reinterpret_cast<float*>(ws + L.aux);
   bool ok = make_map(&mX_k, BF, ra.xhat, d, M, d * 2, 64, kBM) &&
             make_map(&mAux, F32, aux, kBN,
@@ -335,8 +341,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
             make_map(&mW_k, BF, W, d, V, d * 2, 64, kBN / 2) &&
             make_map(&mP_st, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, 32) &&
             make_map(&mG_k, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBM) &&
-            make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK) &&
-            make_map(&mDX, F32, dxhat, d, M, d * 4, 32, 32);
+            make_map(&mW_mn, BF, W, d, V, d * 2, 64, kBK);
   if (ok && dW) {
     ok = make_map(&mG_mn, BF, ra.P, V, M, static_cast<uint64_t>(L.ldp) * 2, 64, kBK) &&
          make_map(&mX_mn, BF, ra.xhat, d, M, d * 2, 64, kBK) &&
@@ -405,13 +410,14 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.dg_part = dgamma ? ra.dgamma_part : nullptr;
   gx.dg_blocks = L.dg_chunks;
   gx.dg_row0 = static_cast<int64_t>(D.K - 1) * D.N;
+  gx.aux_part0 = 1;     // cut tiles: every part to a slot, summed by cut_tiles_norm
   plan_units(gx, sms, true);
-  if (!mark(SOLO_STAGE_DXHAT) ||
-      fail(launch_gemm(kDxhat, mG_k, mW_mn, mDX, mAux, gx, sms, stream)) ||
-      fail(launch_split_fixup(gx, dxhat, D.d, aux, stream)))
+  // whole tiles write dH from TMEM and cut tiles write slots: the output map
+  // is never used (any valid map fills its place)
+  if (!mark(SOLO_STAGE_DXHAT) || fail(launch_gemm(kDxhat, mG_k, mW_mn, mAux, mAux, gx, sms, stream)))
     return SOLO_ERR_CUDA;
 
-  if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_cut_tiles_norm(gx, dxhat, stream)))
+  if (!mark(SOLO_STAGE_NORM_BWD) || fail(launch_cut_tiles_norm(gx, aux, stream)))
     return SOLO_ERR_CUDA;
 
   if (!mark(SOLO_STAGE_DW)) return SOLO_ERR_CUDA;
@@ -425,6 +431,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
     gw.n_blocks = static_cast<int32_t>((d + kBN - 1) / kBN);
     gw.group_m = kGroupDW;
     gw.num_tiles = gw.m_blocks * gw.n_blocks;
+    gw.aux_part0 = 0;
     plan_units(gw, sms, true);
     if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, mAux, gw, sms, stream)) ||
         fail(launch_split_fixup(gw, dW, D.d, aux, stream)))
@@ -770,7 +777,9 @@ const char* solo_readout_strerror(solo_status_t status) {
   switch (status) {
     case SOLO_OK: return "success";
     case SOLO_ERR_INVALID_ARG: return "invalid argument (NULL pointer or dims out of range)";
-    case SOLO_ERR_UNSUPPORTED_SHAPE: return "unsupported shape (d must be a multiple of 8)";
+    case SOLO_ERR_UNSUPPORTED_SHAPE:
+      return "unsupported shape (d must be a multiple of 8; V at most 2^23; K*N and the "
+             "tile counts within 32-bit coordinates)";
     case SOLO_ERR_WORKSPACE_TOO_SMALL: return "workspace smaller than solo_readout_workspace_bytes";
     case SOLO_ERR_CUDA: return "a CUDA runtime call failed";
     case SOLO_ERR_NOT_SM103: return "current device is not compute capability 10.3 (sm_103a)";

@@ -165,6 +165,10 @@ def sampled_check(wl, inp: synth.Inputs, gpu, rows_per_module=24, n_vocab=48, se
         rel = abs(gpu["loss_mean"][k] - want) / abs(want)
         rep["loss_mean_final_rel"] = rel
         assert rel <= LOSS_MEAN_REL, ("loss_mean", k, gpu["loss_mean"][k], want)
+        # every token loss of the final module, element by element
+        err = float(np.max(np.abs(gpu["loss_tok"][k] - ch["loss"])))
+        rep["loss_tok_final_all"] = err
+        assert err <= LOSS_TOK_ABS, ("loss_tok of the final module", err)
         check_grad("dgamma", gpu["dgamma"], ch["dgamma"], rep)
         check_grad("dW rows", gpu["dW"][cols], ch["dW_rows"], rep)
     # each column of dW sums to zero over the vocabulary (rows of G sum to zero)

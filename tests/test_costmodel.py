@@ -51,3 +51,14 @@ def test_call_flops_is_2k_plus_1_readouts():
     # one call over K modules of N tokens = N tokens of the table's readout column
     per_tok = costmodel.per_token_gflops(24, 2048, 4, 2, 2048, 32000)["readouts"] * 1e9
     assert abs(costmodel.call_flops(4, 8192, 2048, 32000) - per_tok * 8192) < 1.0
+
+
+def test_kept_call_flops():
+    """All tokens kept: the call's (2K+1) 2NVd; a masked token of an auxiliary
+    module removes 4Vd, one of the final module 6Vd."""
+    K, N, d, V = 4, 100, 64, 1000
+    assert costmodel.kept_call_flops([N] * K, d, V) == costmodel.call_flops(K, N, d, V)
+    assert costmodel.kept_call_flops([N - 1] + [N] * (K - 1), d, V) == \
+        costmodel.call_flops(K, N, d, V) - 4 * V * d
+    assert costmodel.kept_call_flops([N] * (K - 1) + [N - 1], d, V) == \
+        costmodel.call_flops(K, N, d, V) - 6 * V * d

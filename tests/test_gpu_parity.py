@@ -59,6 +59,38 @@ def test_ragged_shapes(wl):
     parity.compare_full(wl, gpu, ref)
 
 
+# Every GEMM runs several work units per CTA pair here (76 pairs on GB300), so
+# the second TMEM accumulator, its phase flips and raster groups beyond the
+# first are compared element by element:
+#  - 4096 x 2 tokens, d = 1024, V = 8192: logits 32 x 32 = 1024 tiles, dX̂ 32 x 4 =
+#    128 tiles (36 + 52 cut into 2 parts), dW 32 x 4 = 128 tiles;
+#  - 3000 x 3 tokens, d = 776, V = 5000 (no dimension a multiple of 256): logits
+#    36 x 20 = 720 tiles, dX̂ 36 x 4 = 144, dW 20 x 4 = 80 (4 tiles cut into 8).
+MULTIWAVE = [
+    Workload("k2_n4096_d1024_v8192_rowscale_zipf_mask10", K=2, N=4096, d=1024, V=8192,
+             seed=51, targets="zipf", mask_frac=0.1, row_scale=True),
+    Workload("k3_n3000_d776_v5000_heavy_mask5", K=3, N=3000, d=776, V=5000, seed=52,
+             heavy_frac=0.01, mask_frac=0.05, row_scale=True),
+]
+
+
+@pytest.mark.parametrize("wl", MULTIWAVE, ids=lambda w: w.name)
+def test_multiwave_full_parity(wl):
+    """Element-by-element parity where every persistent GEMM loops over many
+    tiles per CTA pair (both accumulators, raster groups, cut last waves)."""
+    import torch
+    from paper_2609_35440_gb300 import solo_readout as sr
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    pairs = sms // 2
+    tiles = lambda rows, cols: -(-rows // 256) * -(-cols // 256)
+    assert tiles(wl.M, wl.V) > 4 * pairs and tiles(wl.M, wl.d) > pairs
+    assert tiles(wl.V, wl.d) > pairs
+    _, gpu, ref = _case(wl)
+    assert gpu["flags"] == 0
+    rep = parity.compare_full(wl, gpu, ref)
+    print(wl.name, rep)
+
+
 def test_mask_array_and_bad_targets():
     wl = Workload("masked_k2_n160_d128_v700", K=2, N=160, d=128, V=700, seed=41)
     inp = synth.generate(wl)
