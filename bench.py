@@ -64,10 +64,12 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=25.0)
-    p.add_argument("--mode", default="train", choices=["train", "heads", "exit", "private"],
+    p.add_argument("--mode", default="train",
+                   choices=["train", "heads", "exit", "private", "onchip"],
                    help="train: forward + backward (the headline); heads: the same with "
                         "each head's temperature and bias and their gradients; exit: "
-                        "forward-only early-exit readout (losses, top-1)")
+                        "forward-only early-exit readout (losses, top-1); onchip: the "
+                        "forward + backward with the auxiliary modules' logits kept on chip")
     return p.parse_args()
 
 
@@ -425,7 +427,10 @@ def run_ours(args, wl):
     hidden = [to_dev(inp.hidden[k]) for k in range(wl.K)]
     gamma, W = to_dev(inp.gamma), to_dev(inp.W)
     targets = torch.from_numpy(inp.targets).to(dev)
-    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index, device=dev)
+    onchip = args.mode == "onchip"
+    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index, device=dev,
+                    onchip=onchip)
+    n_stages = sr.SOLO_ONCHIP_NUM_STAGES if onchip else sr.SOLO_NUM_STAGES
     heads = {}
     if args.mode == "heads":
         tau, bias = synth.gen_heads(wlr)
@@ -444,7 +449,7 @@ def run_ours(args, wl):
 
     # ---- device-resident timing of exactly `steps` calls; events recorded on the
     # launching stream between the stages of every call (read after the loop)
-    step_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(sr.SOLO_NUM_STAGES + 1)]
+    step_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_stages + 1)]
                 for _ in range(args.steps)]
     for evl in step_evs:
         for e in evl:
@@ -463,9 +468,9 @@ def run_ours(args, wl):
     clk.__exit__(None, None, None)
     flags = ro.flags(stream)
     ms = t0.elapsed_time(t1)
-    stage_ms = np.zeros(sr.SOLO_NUM_STAGES)
+    stage_ms = np.zeros(n_stages)
     for evl in step_evs:
-        stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(sr.SOLO_NUM_STAGES)]
+        stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(n_stages)]
     stage_ms /= args.steps
 
     ms = max_over_ranks(ms, dev)
@@ -506,13 +511,19 @@ def run_ours(args, wl):
 
     peaks, peak_src = load_peaks()
     G = costmodel.gemm_flops(wl.M, wl.V, wl.d)     # one module-GEMM over all K modules
-    names = sr.STAGE_NAMES
-    gemm_stage_flops = {"logits": G, "dxhat": G, "dW": G / wl.K}
+    if onchip:
+        names = sr.ONCHIP_STAGE_NAMES
+        # final module: logits, dX and dW over its N tokens; auxiliary modules: the
+        # logits and sum_v P_v W_v of K-1 modules in one pass
+        gemm_stage_flops = {"final": 3 * G / wl.K, "aux_onchip": 2 * G * (wl.K - 1) / wl.K}
+    else:
+        names = sr.STAGE_NAMES
+        gemm_stage_flops = {"logits": G, "dxhat": G, "dW": G / wl.K}
     dom = max(gemm_stage_flops, key=lambda s: stage_ms[names.index(s)])
     dom_ms = stage_ms[names.index(dom)]
     achieved = gemm_stage_flops[dom] / (dom_ms / 1e3) / 1e12
     peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
-    traffic = committed_traffic(wl) if dom == "logits" else None
+    traffic = committed_traffic(wl) if dom == "logits" and not onchip else None
     algo = costmodel.call_flops(wl.K, wl.N, wl.d, wl.V)
     kept = costmodel.kept_call_flops(kept_counts(wl, inp.targets), wl.d, wl.V)
     step_s = ms / 1e3 / args.steps
@@ -521,6 +532,7 @@ def run_ours(args, wl):
         cpu = cpu_baseline(wl, args.cpu_seconds)
     line = {
         "metric": HEADS_METRIC if heads else METRIC, "value": value, "unit": "tokens/s",
+        "workspace_bytes": int(ro.workspace.numel()),
         "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
@@ -539,7 +551,10 @@ def run_ours(args, wl):
         # are recomputed (the forward stores its exponentials)
         "executed_tflops": algo / step_s / 1e12,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
-        "roofline": {"bound": "tensor", "kernel": f"{dom} GEMM (tcgen05)",
+        "roofline": {"bound": "tensor",
+                     "kernel": ("auxiliary on-chip pass (tcgen05, cluster split of d)"
+                                if dom == "aux_onchip" else f"{dom} GEMM (tcgen05)"
+                                if not onchip else "final module, stored path (tcgen05)"),
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": peak_name},

@@ -312,6 +312,58 @@ solo_status_t solo_readout_fwd_bwd_private(const solo_dims_t* dims,
                                            void* workspace, size_t workspace_bytes,
                                            solo_stream_t stream);
 
+/* Stages of the on-chip variant, for solo_readout_fwd_bwd_onchip's events. */
+enum {
+  SOLO_ONCHIP_STAGE_FINAL = 0,     /* the final module on the stored path (all its
+                                      products, dW and dgamma)                     */
+  SOLO_ONCHIP_STAGE_AUX_PREP = 1,  /* auxiliary modules: RMSNorm and kept counts   */
+  SOLO_ONCHIP_STAGE_AUX = 2,       /* auxiliary modules: the single on-chip pass   */
+  SOLO_ONCHIP_STAGE_AUX_MEANS = 3, /* auxiliary modules' mean losses               */
+  SOLO_ONCHIP_NUM_STAGES = 4
+};
+
+/*
+ * The same forward + backward as solo_readout_fwd_bwd, with the auxiliary
+ * modules (0 .. K-2) computed in one pass whose logits never leave the chip
+ * (paper, Section 2.2, Eq. 2-3: the local loss and its readout factor
+ * W-bar^T delta_k).  Per token, with the reference m = a running row maximum,
+ *     dxhat = ((sum over v != y of e^{z_v - m} W_v) / S - (S'/S) W_y) / Nvalid,
+ *     S' = sum over v != y of e^{z_v - m},  S = S' + e^{z_y - m},
+ * and loss = lse - z_y with lse = m + ln S, accumulated over 128-column
+ * vocabulary tiles: each cluster of CTAs keeps a 128-row block's slice of
+ * xhat, its partial logits, the exponentials P and sum_v P_v W_v in tensor
+ * and shared memory.  Nothing of size tokens x vocabulary is written for
+ * these modules, so their workspace is xhat and a few floats per token.  The
+ * final module, whose dW needs the whole logit gradient, takes the stored path
+ * of solo_readout_fwd_bwd over its own N tokens.
+ *
+ * Arguments and outputs are those of solo_readout_fwd_bwd; the workspace is
+ * solo_readout_onchip_workspace_bytes (the final module's stored-path
+ * workspace for N tokens plus K-1 modules' xhat, r and token losses).
+ * events: NULL, or SOLO_ONCHIP_NUM_STAGES + 1 cudaEvent_t handles, recorded
+ * before each stage and after the last (n_events must then be
+ * SOLO_ONCHIP_NUM_STAGES + 1).  Widths above 2048 are refused with
+ * SOLO_ERR_UNSUPPORTED_SHAPE (a 128-row block's accumulator would need more
+ * than the 8 CTAs of a portable cluster).  Results agree with
+ * solo_readout_fwd_bwd within the parity tolerances, not bit for bit (the
+ * exponentials are formed against a different reference).
+ */
+solo_status_t solo_readout_onchip_workspace_bytes(const solo_dims_t* dims, size_t* bytes);
+solo_status_t solo_readout_fwd_bwd_onchip(const solo_dims_t* dims,
+                                          const solo_bf16_t* const* hidden,
+                                          const solo_bf16_t* gamma,
+                                          const solo_bf16_t* W,
+                                          const int32_t* targets,
+                                          const uint8_t* mask,
+                                          float* loss_tok,
+                                          float* loss_mean,
+                                          solo_bf16_t* const* dhidden,
+                                          float* dW,
+                                          float* dgamma,
+                                          void* workspace, size_t workspace_bytes,
+                                          solo_stream_t stream,
+                                          void* const* events, int32_t n_events);
+
 /*
  * The final RMSNorm alone (the first step of every call): for each module k
  * and token i, r_i = (mean_j h_ij^2 + eps)^-1/2 and xhat_ij = bf16(gamma_j

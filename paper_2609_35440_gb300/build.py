@@ -19,7 +19,7 @@ LIB = os.path.join(LIBDIR, "libsolo_readout.so")
 # The checked build: every computed global index of the row kernels and GEMM
 # epilogues is tested (SOLO_DEBUG=1); a violation sets SOLO_FLAG_BOUNDS.
 LIB_CHECKED = os.path.join(LIBDIR, "libsolo_readout_checked.so")
-SOURCES = ["gemm_tc.cu", "rowops.cu", "solo_readout.cu", "selftest.cu"]
+SOURCES = ["gemm_tc.cu", "rowops.cu", "solo_readout.cu", "selftest.cu", "flash_bwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr"]

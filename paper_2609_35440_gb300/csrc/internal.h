@@ -151,6 +151,54 @@ cudaError_t launch_split_fixup(const GemmArgs& g, float* out, int64_t ld, const 
 // buffer, added in part order.
 cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* aux, cudaStream_t stream);
 
+// ---- single-pass on-chip backward of the auxiliary modules ------------------------
+// dxhat_i = (sum over v != y of exp(z_v - m) W_v) / S - (S' / S) W_y (Eq. 3 with the
+// softmax written out; S = sum over all v of exp(z_v - m), S' the same without the
+// target), accumulated over the vocabulary with the logits kept on chip.  A
+// cluster of C CTAs shares a block of 128 rows; CTA c owns the d-columns
+// [c * ds, c * ds + ds) of dxhat.
+
+struct FlashArgs {
+  int32_t M;             // auxiliary rows (K - 1 modules of N tokens, module-major)
+  int32_t d;
+  int32_t V;
+  int32_t ds;            // d-columns per CTA (multiple of 64, <= 256)
+  int32_t n_tiles;       // 128-column vocabulary tiles
+  int32_t row_blocks;    // 128-row blocks
+  int64_t N;             // tokens per module
+  int32_t modules;       // auxiliary modules (K - 1)
+  int32_t ignore_index;
+  const int32_t* targets;   // [M]
+  const uint8_t* mask;      // [M] or null
+  const uint16_t* xhat;     // [M, d] bf16
+  const float* r;           // [M]
+  const float* inv_nvalid;  // [modules]
+  const uint16_t* W;        // [V, d] bf16
+  const uint16_t* gamma;    // [d]
+  const uint16_t* hidden[kMaxModules];
+  uint16_t* dhidden[kMaxModules];
+  float* loss_tok;          // [M] or null
+  float* row_loss;          // [M]: token loss (0 when masked), for the module means
+  int32_t* n_valid;         // [modules]
+  float* loss_mean;         // [modules]
+  uint32_t* flags;
+};
+
+// Largest width the on-chip backward handles: 8 CTAs of 256 columns.
+constexpr int kFlashMaxD = 2048;
+// CTAs per cluster (1, 2, 4 or 8) and d-columns per CTA (a multiple of 64) for width d.
+int flash_cluster_size(int d);
+int flash_slice_width(int d);
+cudaError_t flash_prepare(int device);
+// Kept-token counts and 1/Nvalid of the auxiliary modules (and bad-target flags).
+cudaError_t launch_flash_count(const FlashArgs& a, float* inv_nvalid, cudaStream_t s);
+// The on-chip forward + backward of the auxiliary rows; w: tensor map of W
+// (bf16 [V, d], 64 x 128 boxes, 128-byte swizzle).
+cudaError_t launch_flash(const CUtensorMap& w, const FlashArgs& a, int device, int sms,
+                         cudaStream_t s);
+// Module means of the auxiliary modules from row_loss, in a fixed order.
+cudaError_t launch_flash_means(const FlashArgs& a, cudaStream_t s);
+
 // ---- row kernels ---------------------------------------------------------------
 
 struct RowArgs {

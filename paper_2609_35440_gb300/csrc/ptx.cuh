@@ -1,5 +1,7 @@
 // Inline-PTX wrappers for sm_103a: mbarrier, TMA (cp.async.bulk.tensor),
-// tcgen05 (TMEM allocation, MMA, commit, loads) and bounded waits.
+// cluster shared-memory transfers (st.async, bulk copies), tcgen05 (TMEM
+// allocation, MMA with A in shared or tensor memory, commit, loads, stores) and
+// bounded waits.
 #pragma once
 
 #include <cstdint>
@@ -127,6 +129,43 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t saddr, uint32_t rank) {
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                : "memory");
+}
+
+// Stores 16 bytes into shared memory of a CTA of the cluster (a shared::cluster
+// address from map_to_rank) and completes that many transaction bytes on the
+// mbarrier at bar_cluster (same CTA as the data).
+__device__ __forceinline__ void st_async_v4(uint32_t addr_cluster, uint32_t a, uint32_t b,
+                                            uint32_t c, uint32_t d, uint32_t bar_cluster) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];"
+      ::"r"(addr_cluster), "r"(a), "r"(b), "r"(c), "r"(d), "r"(bar_cluster)
+      : "memory");
+}
+
+// Bulk copy (async proxy) of `bytes` (a multiple of 16, both addresses 16-byte
+// aligned) from this CTA's shared memory to a CTA of the cluster; completes the
+// bytes on the destination CTA's mbarrier at bar_cluster.
+__device__ __forceinline__ void bulk_copy_s2s(uint32_t dst_cluster, uint32_t src_cta,
+                                              uint32_t bytes, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst_cluster), "r"(src_cta), "r"(bytes), "r"(bar_cluster)
+      : "memory");
+}
+
+// bar.red.and over `count` threads of named barrier `id`: every participant
+// gets the AND of their predicates.
+__device__ __forceinline__ bool named_bar_and(uint32_t id, uint32_t count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
 }
 
 __device__ __forceinline__ void cluster_sync() {
@@ -269,6 +308,30 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
       : "memory");
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]: A in tensor memory (row i in lane i, two
+// bf16 per 32-bit column, K = 16 per instruction = 8 columns), bf16 inputs,
+// fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives once on the barrier at this shared-memory offset in every CTA of
+// `cta_mask` when all tcgen05 operations this thread issued so far have
+// completed (single-CTA MMAs).
+__device__ __forceinline__ void mma_commit_multicast(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(cta_mask)
+      : "memory");
+}
+
 // Arrives once on `bar` when all tcgen05 operations this thread issued so far
 // have completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -298,6 +361,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
       : "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 consecutive 32-bit columns of this warp's 32 TMEM lanes from registers
+// (lane i of the warp writes TMEM lane base + i); waits for the stores.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
 }
 
 // ---- descriptors -------------------------------------------------------------

@@ -165,7 +165,7 @@ struct DeviceInfo {
 std::mutex g_dev_mu;
 DeviceInfo g_dev[64];
 
-solo_status_t device_setup(int* sms) {
+solo_status_t device_setup(int* sms, int* device = nullptr) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return SOLO_ERR_CUDA;
   if (dev < 0 || dev >= 64) return SOLO_ERR_CUDA;
@@ -179,11 +179,13 @@ solo_status_t device_setup(int* sms) {
       return SOLO_ERR_CUDA;
     info.sm103 = (major == 10 && minor == 3);
     info.sms = sms_;
-    if (info.sm103 && gemm_prepare(dev) != cudaSuccess) return SOLO_ERR_CUDA;
+    if (info.sm103 && (gemm_prepare(dev) != cudaSuccess || flash_prepare(dev) != cudaSuccess))
+      return SOLO_ERR_CUDA;
     info.ready = true;
   }
   if (!info.sm103) return SOLO_ERR_NOT_SM103;
   *sms = info.sms;
+  if (device) *device = dev;
   return SOLO_OK;
 }
 
@@ -586,9 +588,189 @@ solo_status_t run_exit(const solo_dims_t* dims, const solo_bf16_t* const* hidden
   return SOLO_OK;
 }
 
+// ---- on-chip backward of the auxiliary modules ----------------------------------
+
+struct OnchipLayout {
+  size_t final_total = 0;     // the final module's stored-path layout, at offset 0
+  size_t xhat = 0, r = 0, row_loss = 0, n_valid = 0, inv_nvalid = 0, total = 0;
+};
+
+OnchipLayout make_onchip_layout(const solo_dims_t& d) {
+  OnchipLayout L;
+  solo_dims_t one = d;
+  one.K = 1;
+  L.final_total = make_layout(one).total;
+  const size_t Maux = static_cast<size_t>(d.K - 1) * static_cast<size_t>(d.N);
+  size_t off = align_up(L.final_total, kAlign);
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes, kAlign);
+    return at;
+  };
+  L.xhat = take(Maux * d.d * 2);
+  L.r = take(Maux * 4);
+  L.row_loss = take(Maux * 4);
+  L.n_valid = take(SOLO_MAX_MODULES * 4);
+  L.inv_nvalid = take(SOLO_MAX_MODULES * 4);
+  L.total = off;
+  return L;
+}
+
+solo_status_t check_onchip_dims(const solo_dims_t* dims) {
+  const solo_status_t st = check_dims(dims);
+  if (st != SOLO_OK) return st;
+  if (dims->d > kFlashMaxD) return SOLO_ERR_UNSUPPORTED_SHAPE;
+  return SOLO_OK;
+}
+
+solo_status_t run_onchip(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
+                         const solo_bf16_t* gamma, const solo_bf16_t* W, const int32_t* targets,
+                         const uint8_t* mask, float* loss_tok, float* loss_mean,
+                         solo_bf16_t* const* dhidden, float* dW, float* dgamma, void* workspace,
+                         size_t workspace_bytes, cudaStream_t stream, void* const* events,
+                         int32_t n_events) {
+  solo_status_t st = check_onchip_dims(dims);
+  if (st != SOLO_OK) return st;
+  const solo_dims_t& D = *dims;
+  if (hidden == nullptr || dhidden == nullptr || gamma == nullptr || W == nullptr ||
+      targets == nullptr || loss_mean == nullptr || workspace == nullptr)
+    return SOLO_ERR_INVALID_ARG;
+  if (events != nullptr && n_events != SOLO_ONCHIP_NUM_STAGES + 1) return SOLO_ERR_INVALID_ARG;
+  for (int k = 0; k < D.K; ++k) {
+    if (hidden[k] == nullptr || dhidden[k] == nullptr) return SOLO_ERR_INVALID_ARG;
+    if (!aligned16(hidden[k]) || !aligned16(dhidden[k])) return SOLO_ERR_MISALIGNED;
+  }
+  if (!aligned16(gamma) || !aligned16(W) || !aligned16(workspace) ||
+      (reinterpret_cast<uintptr_t>(targets) & 3u) || (dW && !aligned16(dW)) ||
+      (dgamma && (reinterpret_cast<uintptr_t>(dgamma) & 3u)) ||
+      (loss_tok && (reinterpret_cast<uintptr_t>(loss_tok) & 3u)) ||
+      (reinterpret_cast<uintptr_t>(loss_mean) & 3u))
+    return SOLO_ERR_MISALIGNED;
+  const OnchipLayout L = make_onchip_layout(D);
+  if (workspace_bytes < L.total) return SOLO_ERR_WORKSPACE_TOO_SMALL;
+  {
+    const size_t K = static_cast<size_t>(D.K), N = static_cast<size_t>(D.N);
+    const size_t dd = static_cast<size_t>(D.d), VV = static_cast<size_t>(D.V);
+    Ranges rg;
+    for (int k = 0; k < D.K; ++k) {
+      rg.add(hidden[k], N * dd * 2, false);
+      rg.add(dhidden[k], N * dd * 2, true);
+    }
+    rg.add(gamma, dd * 2, false);
+    rg.add(W, VV * dd * 2, false);
+    rg.add(targets, K * N * 4, false);
+    rg.add(mask, K * N, false);
+    rg.add(loss_tok, K * N * 4, true);
+    rg.add(loss_mean, K * 4, true);
+    rg.add(dW, VV * dd * 4, true);
+    rg.add(dgamma, dd * 4, true);
+    rg.add(workspace, L.total, true);
+    if (rg.any_output_overlap()) return SOLO_ERR_INVALID_ARG;
+  }
+  int sms = 0, dev = 0;
+  st = device_setup(&sms, &dev);
+  if (st != SOLO_OK) return st;
+  auto mark = [&](int stage) -> bool {
+    if (events == nullptr) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(events[stage]), stream) == cudaSuccess;
+  };
+
+  // 1. the final module on the stored path (it needs G for dW); clears the flags
+  const int64_t kf = D.K - 1;
+  solo_dims_t one = D;
+  one.K = 1;
+  if (!mark(SOLO_ONCHIP_STAGE_FINAL)) return SOLO_ERR_CUDA;
+  st = run(&one, hidden + kf, gamma, W, targets + kf * D.N, mask ? mask + kf * D.N : nullptr,
+           nullptr, loss_tok ? loss_tok + kf * D.N : nullptr, loss_mean + kf, dhidden + kf, dW,
+           dgamma, workspace, L.final_total, stream, nullptr, 0, /*clear_flags=*/true);
+  if (st != SOLO_OK) return st;
+
+  // 2. the auxiliary modules in one on-chip pass
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const int aux = D.K - 1;
+  FlashArgs fa;
+  std::memset(&fa, 0, sizeof(fa));
+  fa.M = static_cast<int32_t>(static_cast<int64_t>(aux) * D.N);
+  fa.d = D.d;
+  fa.V = D.V;
+  fa.ds = flash_slice_width(D.d);
+  fa.n_tiles = (D.V + 127) / 128;
+  fa.row_blocks = static_cast<int32_t>((static_cast<int64_t>(fa.M) + 127) / 128);
+  fa.N = D.N;
+  fa.modules = aux;
+  fa.ignore_index = D.ignore_index;
+  fa.targets = targets;
+  fa.mask = mask;
+  fa.xhat = reinterpret_cast<const uint16_t*>(ws + L.xhat);
+  fa.r = reinterpret_cast<const float*>(ws + L.r);
+  float* inv_nvalid = reinterpret_cast<float*>(ws + L.inv_nvalid);
+  fa.inv_nvalid = inv_nvalid;
+  fa.W = W;
+  fa.gamma = gamma;
+  for (int k = 0; k < aux; ++k) {
+    fa.hidden[k] = hidden[k];
+    fa.dhidden[k] = dhidden[k];
+  }
+  fa.loss_tok = loss_tok;
+  fa.row_loss = reinterpret_cast<float*>(ws + L.row_loss);
+  fa.n_valid = reinterpret_cast<int32_t*>(ws + L.n_valid);
+  fa.loss_mean = loss_mean;
+  fa.flags = reinterpret_cast<uint32_t*>(ws);     // the final module's flag word
+  if (!mark(SOLO_ONCHIP_STAGE_AUX_PREP)) return SOLO_ERR_CUDA;
+  CUtensorMap mW;
+  if (aux > 0) {
+    RowArgs ra;
+    std::memset(&ra, 0, sizeof(ra));
+    for (int k = 0; k < aux; ++k) ra.hidden[k] = hidden[k];
+    ra.N = D.N;
+    ra.K = aux;
+    ra.d = D.d;
+    ra.V = D.V;
+    ra.eps = D.eps;
+    ra.gamma = gamma;
+    ra.xhat = reinterpret_cast<uint16_t*>(ws + L.xhat);
+    ra.r = reinterpret_cast<float*>(ws + L.r);
+    ra.flags = fa.flags;
+    if (launch_rmsnorm_fwd(ra, stream) != cudaSuccess ||
+        launch_flash_count(fa, inv_nvalid, stream) != cudaSuccess)
+      return SOLO_ERR_CUDA;
+    if (!make_map(&mW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, W, static_cast<uint64_t>(D.d),
+                  static_cast<uint64_t>(D.V), static_cast<uint64_t>(D.d) * 2, 64, 128))
+      return SOLO_ERR_CUDA;
+  }
+  if (!mark(SOLO_ONCHIP_STAGE_AUX)) return SOLO_ERR_CUDA;
+  if (aux > 0 && launch_flash(mW, fa, dev, sms, stream) != cudaSuccess) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_ONCHIP_STAGE_AUX_MEANS)) return SOLO_ERR_CUDA;
+  if (aux > 0 && launch_flash_means(fa, stream) != cudaSuccess) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_ONCHIP_NUM_STAGES)) return SOLO_ERR_CUDA;
+  return SOLO_OK;
+}
+
 }  // namespace
 
 extern "C" {
+
+solo_status_t solo_readout_onchip_workspace_bytes(const solo_dims_t* dims, size_t* bytes) {
+  if (bytes == nullptr) return SOLO_ERR_INVALID_ARG;
+  const solo_status_t st = check_onchip_dims(dims);
+  if (st != SOLO_OK) return st;
+  *bytes = make_onchip_layout(*dims).total;
+  return SOLO_OK;
+}
+
+solo_status_t solo_readout_fwd_bwd_onchip(const solo_dims_t* dims,
+                                          const solo_bf16_t* const* hidden,
+                                          const solo_bf16_t* gamma, const solo_bf16_t* W,
+                                          const int32_t* targets, const uint8_t* mask,
+                                          float* loss_tok, float* loss_mean,
+                                          solo_bf16_t* const* dhidden, float* dW, float* dgamma,
+                                          void* workspace, size_t workspace_bytes,
+                                          solo_stream_t stream, void* const* events,
+                                          int32_t n_events) {
+  return run_onchip(dims, hidden, gamma, W, targets, mask, loss_tok, loss_mean, dhidden, dW,
+                    dgamma, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream),
+                    events, events ? n_events : 0);
+}
 
 solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* bytes) {
   if (bytes == nullptr) return SOLO_ERR_INVALID_ARG;

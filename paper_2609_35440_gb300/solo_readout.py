@@ -29,6 +29,8 @@ SOLO_FLAG_TIMEOUT = 2
 
 SOLO_NUM_STAGES = 8
 SOLO_EXIT_NUM_STAGES = 3
+SOLO_ONCHIP_NUM_STAGES = 4
+ONCHIP_STAGE_NAMES = ["final", "aux_prep", "aux_onchip", "aux_means"]
 EXIT_STAGE_NAMES = ["rmsnorm", "logits", "combine"]
 STAGE_NAMES = ["rmsnorm", "logits", "lse", "grad", "dxhat", "norm_bwd", "dW", "dgamma"]
 
@@ -117,6 +119,10 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.solo_readout_build_flags.restype = i32
     lib.solo_readout_rmsnorm.argtypes = [dims_p, ctypes.POINTER(vp), vp, vp, vp, vp]
     lib.solo_readout_rmsnorm.restype = i32
+    lib.solo_readout_onchip_workspace_bytes.argtypes = [dims_p, ctypes.POINTER(sz)]
+    lib.solo_readout_onchip_workspace_bytes.restype = i32
+    lib.solo_readout_fwd_bwd_onchip.argtypes = common + [ctypes.POINTER(vp), i32]
+    lib.solo_readout_fwd_bwd_onchip.restype = i32
     _lib = lib
     return lib
 
@@ -336,6 +342,33 @@ def solo_readout_fwd_bwd_private(dims: solo_dims_t, hidden: Sequence, gammas: Se
     return st
 
 
+def solo_readout_onchip_workspace_bytes(dims: solo_dims_t) -> int:
+    out = ctypes.c_size_t(0)
+    st = load().solo_readout_onchip_workspace_bytes(ctypes.byref(dims), ctypes.byref(out))
+    if st != SOLO_OK:
+        raise SoloError(st, "solo_readout_onchip_workspace_bytes")
+    return out.value
+
+
+def solo_readout_fwd_bwd_onchip(dims: solo_dims_t, hidden: Sequence, gamma, W, targets, mask,
+                                loss_tok, loss_mean, dhidden: Sequence, dW, dgamma, workspace,
+                                workspace_bytes: int | None = None, stream=None, events=None,
+                                check: bool = True) -> int:
+    """The call with the auxiliary modules' logits kept on chip (events: None or
+    SOLO_ONCHIP_NUM_STAGES + 1 torch.cuda.Event around its stages)."""
+    if events is None:
+        extra = (None, 0)
+    else:
+        handles = [e.cuda_event if hasattr(e, "cuda_event") else int(e) for e in events]
+        extra = ((ctypes.c_void_p * len(handles))(*handles), len(handles))
+    st = _call(load().solo_readout_fwd_bwd_onchip, dims, hidden, gamma, W, targets, mask,
+               loss_tok, loss_mean, dhidden, dW, dgamma, workspace, workspace_bytes, stream,
+               extra=extra)
+    if check and st != SOLO_OK:
+        raise SoloError(st, "solo_readout_fwd_bwd_onchip")
+    return st
+
+
 def solo_readout_get_flags(workspace, stream=None) -> int:
     out = ctypes.c_uint32(0)
     st = load().solo_readout_get_flags(_ptr(workspace), _stream_handle(stream), ctypes.byref(out))
@@ -382,15 +415,19 @@ def solo_readout_kernel_launches() -> int:
 
 
 class Readout:
-    """Owns the output and workspace tensors for one problem size (torch, one device)."""
+    """Owns the output and workspace tensors for one problem size (torch, one device).
+    onchip=True selects solo_readout_fwd_bwd_onchip (the auxiliary modules' logits
+    kept on chip) for calls without the heads' parameters."""
 
     def __init__(self, K: int, N: int, d: int, V: int, eps: float = 1e-6,
                  ignore_index: int = -100, want_loss_tok: bool = True, want_dW: bool = True,
-                 want_dgamma: bool = True, device=None):
+                 want_dgamma: bool = True, device=None, onchip: bool = False):
         import torch
         self.dims = make_dims(K, N, d, V, eps, ignore_index)
+        self.onchip = onchip
         dev = torch.device("cuda" if device is None else device)
-        nbytes = solo_readout_workspace_bytes(self.dims)
+        nbytes = (solo_readout_onchip_workspace_bytes(self.dims) if onchip
+                  else solo_readout_workspace_bytes(self.dims))
         self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
         self.loss_tok = torch.empty(K, N, dtype=torch.float32, device=dev) if want_loss_tok else None
         self.loss_mean = torch.empty(K, dtype=torch.float32, device=dev)
@@ -404,7 +441,14 @@ class Readout:
                  tau=None, bias=None, head_grads=False):
         """tau [K] / bias [K, V] (fp32, either may be None) select the heads' call;
         head_grads also fills self.dtau and self.dbias."""
-        if tau is not None or bias is not None or head_grads:
+        if self.onchip:
+            if tau is not None or bias is not None or head_grads:
+                raise ValueError("the on-chip call takes no heads' parameters")
+            solo_readout_fwd_bwd_onchip(self.dims, hidden, gamma, W, targets, mask,
+                                        self.loss_tok, self.loss_mean, self.dhidden, self.dW,
+                                        self.dgamma, self.workspace, stream=stream,
+                                        events=events)
+        elif tau is not None or bias is not None or head_grads:
             solo_readout_fwd_bwd_heads(self.dims, hidden, gamma, W, targets, mask, tau, bias,
                                        self.dtau if head_grads else None,
                                        self.dbias if head_grads else None, self.loss_tok,

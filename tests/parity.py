@@ -34,7 +34,8 @@ def bf16_tensor_to_f64(t) -> np.ndarray:
 
 
 def run_gpu(wl, inp: synth.Inputs, mask: np.ndarray | None = None, want_dW=True,
-            want_dgamma=True, want_loss_tok=True, targets: np.ndarray | None = None):
+            want_dgamma=True, want_loss_tok=True, targets: np.ndarray | None = None,
+            onchip: bool = False):
     import torch
     from paper_2609_35440_gb300 import solo_readout as sr
     dev = torch.device("cuda")
@@ -45,7 +46,8 @@ def run_gpu(wl, inp: synth.Inputs, mask: np.ndarray | None = None, want_dW=True,
     tgt = torch.from_numpy(np.ascontiguousarray(tg, dtype=np.int32)).to(dev)
     mk = None if mask is None else torch.from_numpy(np.ascontiguousarray(mask, np.uint8)).to(dev)
     ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, ignore_index=wl.ignore_index,
-                    want_loss_tok=want_loss_tok, want_dW=want_dW, want_dgamma=want_dgamma)
+                    want_loss_tok=want_loss_tok, want_dW=want_dW, want_dgamma=want_dgamma,
+                    onchip=onchip)
     ro(hidden, gamma, W, tgt, mk)
     flags = ro.flags()
     torch.cuda.synchronize()
