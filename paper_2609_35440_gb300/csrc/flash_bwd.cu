@@ -14,7 +14,7 @@
 // Layout on GB300: O for 128 rows needs 128 x d fp32, more than the 512 columns
 // of tensor memory once d > 256, so a cluster of C CTAs (C = 1, 2, 4, 8) shares
 // a block of 128 rows and CTA c owns d-columns [c ds, c ds + ds) of O.  Per
-// 128-column vocabulary tile each CTA:
+// 64-column vocabulary tile each CTA:
 //   - multiplies its slice of xhat (kept in tensor memory as the A operand)
 //     by its slice of the W tile: a partial Z, a split of the d-sum;
 //   - sends every row of the partial Z to the CTA that owns the row's
@@ -23,6 +23,13 @@
 //     forms P = bf16(e^{z - m}) and broadcasts its rows of P to the cluster
 //     with bulk copies;
 //   - accumulates O += P W_slice (W tile reused from shared memory, MN-major).
+// Partial Z, P and the owners' receive buffers are double-buffered and the O
+// product of tile t is issued after the partial Z of tile t + 2, so the
+// exchanges of two tiles are in flight while the tensor core works; the
+// exchange (fp32 partials, 7/8 of 32 KB out and in per CTA and tile at C = 8,
+// plus bf16 P) is what bounds the pass: distributed shared memory moves
+// about 15-18 B/clk per SM on GB300 (measured), against 64 B/clk of operands
+// the tensor core reads.
 // The reference m of a row is the maximum of its first tile; it is not moved
 // while the logits stay within 64 of it (e^64 fits fp32 and bf16 with room
 // for V terms).  A row whose maximum exceeds that has its whole block swept a
@@ -47,42 +54,50 @@ namespace solo {
 namespace {
 
 constexpr int kFR = 128;                       // rows per block (tensor-memory lanes)
-constexpr int kFV = 128;                       // vocabulary columns per tile
+constexpr int kFV = 64;                        // vocabulary columns per tile
 constexpr int kFDS = 256;                      // widest d-slice of one CTA
 constexpr int kFThreads = 320;
-constexpr int kFAtom = kFV * 128;              // one 64-column swizzle atom of a W tile (16 KB)
-constexpr int kFStageBytes = kFV * kFDS * 2;   // a W tile slice: 64 KB
-constexpr int kFSmemP = 2 * kFStageBytes;      // two W stages
-constexpr int kFPBytes = kFR * kFV * 2;        // P tile, bf16, K-major, 2 atoms (32 KB)
-constexpr int kFSmemPart = kFSmemP + kFPBytes;
-constexpr int kFPartBytes = kFR * kFV * 4;     // partial Z rows received as owner (64 KB)
-constexpr int kFSmemBar = kFSmemPart + kFPartBytes;
-constexpr int kFNumBars = 15;
+constexpr int kFStages = 4;                    // W tiles in flight
+constexpr int kFLag = 2;                       // tiles the O product trails the partial Z
+constexpr int kFAtom = kFV * 128;              // one 64-column swizzle atom of a W tile (8 KB)
+constexpr int kFStageBytes = kFV * kFDS * 2;   // a W tile slice: 32 KB
+constexpr int kFPBytes = kFR * kFV * 2;        // a P tile: bf16, K-major, one atom (16 KB)
+// Partial-Z rows received as owner, fp32: the 16 quads (16 B) of a row sit at
+// positions quad ^ (row & 15), so that the owners' float4 reads and the senders'
+// stores spread over all banks.
+constexpr int kFPartBytes = kFR * kFV * 4;     // 32 KB
+constexpr int kFSmemP = kFStages * kFStageBytes;
+constexpr int kFSmemPart = kFSmemP + 2 * kFPBytes;
+constexpr int kFSmemBar = kFSmemPart + 2 * kFPartBytes;
+constexpr int kFNumBars = 2 * kFStages + 6 * 2 + 5;
 constexpr int kFSmemMisc = kFSmemBar + kFNumBars * 8;
 constexpr int kFSmemTotal = kFSmemMisc + 32 + 1024;   // + alignment slack
 static_assert(kFSmemTotal <= 232448, "shared memory budget");
 // tensor-memory columns
 constexpr uint32_t kTX = 0;      // xhat slice: ds bf16 = ds / 2 columns
-constexpr uint32_t kTZ = 128;    // partial Z of a tile: 128 columns
+constexpr uint32_t kTZ = 128;    // two partial-Z buffers of 64 columns
 constexpr uint32_t kTO = 256;    // O slice: ds columns
 constexpr float kMoveRef = 64.f; // a logit this far above the reference forces a second sweep
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Barriers ([2] = one per buffer of a double-buffered resource; buffer t & 1
+// serves tile t, and its phase for tile t is (t >> 1) & 1).
 enum Bar {
-  bWfull = 0,     // [2] W stage loaded (TMA bytes)
-  bWempty = 2,    // [2] W stage free (MMA commit after the tile's O product)
-  bZfull = 4,     // partial Z in tensor memory (MMA commit)
-  bZempty = 5,    // partial Z read out (4 lane warps)
-  bXready = 6,    // sweep announced, xhat slice in tensor memory (4 lane warps)
-  bPfull = 7,     // the P tile is complete in this CTA (owner rows: local arrive; others: bytes)
-  bPfree = 8,     // every CTA's O product of the previous tile done (C multicast commits)
-  bPartFull = 9,  // partial Z rows of all C CTAs received (bytes)
-  bPartFree = 10, // every owner consumed this CTA's previous partials (C remote arrives)
-  bOfull = 11,    // O of the sweep complete (MMA commit)
-  bOempty = 12,   // O read out (4 lane warps)
-  bRfull = 13,    // per-row factors of the sweep received (bytes)
-  bDrain = 14
+  bWfull = 0,                    // [kFStages] W stage loaded (TMA bytes)
+  bWempty = bWfull + kFStages,   // [kFStages] W stage free (MMA commit after its O product)
+  bZfull = bWempty + kFStages,   // [2] partial Z in tensor memory (MMA commit)
+  bZempty = bZfull + 2,          // [2] partial Z read out (4 lane warps)
+  bPfull = bZempty + 2,          // [2] P tile complete in this CTA (own rows: arrive; others: bytes)
+  bPfree = bPfull + 2,           // [2] every CTA's O product of the buffer's last tile done
+  bPartFull = bPfree + 2,        // [2] partial-Z rows of all C CTAs received (bytes)
+  bPartFree = bPartFull + 2,     // [2] every owner consumed this CTA's partials of the buffer
+  bXready = bPartFree + 2,       // sweep announced, xhat slice in tensor memory (4 lane warps)
+  bOfull,                        // O of the sweep complete (MMA commit)
+  bOempty,                       // O read out (4 lane warps)
+  bRfull,                        // per-row factors of the sweep received (bytes)
+  bDrain
 };
+static_assert(bDrain + 1 == kFNumBars, "barrier count");
 
 struct SweepInfo {
   int valid;
@@ -111,15 +126,16 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
     flash_bwd_kernel(const __grid_constant__ CUtensorMap tmW, const FlashArgs a) {
   constexpr int R = kFR / C;           // rows whose statistics one CTA owns
   constexpr int TPR = 128 / R;         // owner threads per row
-  constexpr int G8 = R / 8;            // 8-column groups per owner thread and tile
+  constexpr int NQ = 16 / TPR;          // 4-column quads per owner thread and 64-column tile
+  static_assert(NQ >= 1 && TPR * NQ * 4 == kFV, "owner columns");
   constexpr uint16_t kAll = static_cast<uint16_t>((1u << C) - 1u);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* ring = smem;
-  uint8_t* ptile = smem + kFSmemP;
-  uint8_t* part = smem + kFSmemPart;
+  uint8_t* ptiles = smem + kFSmemP;
+  uint8_t* parts = smem + kFSmemPart;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kFSmemBar);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kFSmemMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kFSmemMisc + 4);
@@ -133,17 +149,19 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
   const int col0 = static_cast<int>(rank) * a.ds;    // first d-column of this CTA's slice
 
   if (threadIdx.x == 0) {
-    mbar_init(&bars[bWfull], 1);
-    mbar_init(&bars[bWfull + 1], 1);
-    mbar_init(&bars[bWempty], 1);
-    mbar_init(&bars[bWempty + 1], 1);
-    mbar_init(&bars[bZfull], 1);
-    mbar_init(&bars[bZempty], 4);
+    for (int i = 0; i < kFStages; ++i) {
+      mbar_init(&bars[bWfull + i], 1);
+      mbar_init(&bars[bWempty + i], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars[bZfull + b], 1);
+      mbar_init(&bars[bZempty + b], 4);
+      mbar_init(&bars[bPfull + b], 1);
+      mbar_init(&bars[bPfree + b], C);
+      mbar_init(&bars[bPartFull + b], 1);
+      mbar_init(&bars[bPartFree + b], C);
+    }
     mbar_init(&bars[bXready], 4);
-    mbar_init(&bars[bPfull], 1);
-    mbar_init(&bars[bPfree], C);
-    mbar_init(&bars[bPartFull], 1);
-    mbar_init(&bars[bPartFree], C);
     mbar_init(&bars[bOfull], 1);
     mbar_init(&bars[bOempty], 4);
     mbar_init(&bars[bRfull], 1);
@@ -164,11 +182,12 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
   // Initial phases: no owner holds partials and no P tile is in use yet, so
   // each CTA completes phase 0 of every CTA's "partials free" and "P free".
   if (threadIdx.x == 192) {
-    for (int c = 0; c < C; ++c) {
-      mbar_arrive_remote(map_to_rank(smem_u32(&bars[bPartFree]), c));
-      mbar_arrive_remote(map_to_rank(smem_u32(&bars[bPfree]), c));
-    }
-    mbar_arrive_expect_tx(&bars[bPartFull], C * R * kFV * 4);
+    for (int c = 0; c < C; ++c)
+      for (int b = 0; b < 2; ++b) {
+        mbar_arrive_remote(map_to_rank(smem_u32(&bars[bPartFree + b]), c));
+        mbar_arrive_remote(map_to_rank(smem_u32(&bars[bPfree + b]), c));
+      }
+    for (int b = 0; b < 2; ++b) mbar_arrive_expect_tx(&bars[bPartFull + b], C * R * kFV * 4);
   }
   if (threadIdx.x == 64) mbar_arrive_expect_tx(&bars[bRfull], kFR * 16);
 
@@ -182,8 +201,8 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
         if (!(ok = mbar_wait(&bars[bXready], s & 1, abort_flag))) break;
         if (!info->valid) break;
         for (int j = 0; j < a.n_tiles; ++j, ++t) {
-          const int st = t & 1;
-          const uint32_t ph = (t >> 1) & 1;
+          const int st = t % kFStages;
+          const uint32_t ph = (t / kFStages) & 1;
           if (!(ok = mbar_wait(&bars[bWempty + st], ph ^ 1, abort_flag))) break;
           mbar_arrive_expect_tx(&bars[bWfull + st], bytes);
           for (int at = 0; at < a.ds / 64; ++at)
@@ -195,7 +214,7 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
       }
       if (!ok) {
         atomicOr(a.flags, SOLO_FLAG_TIMEOUT);
-        for (int st = 0; st < 2; ++st)
+        for (int st = 0; st < kFStages; ++st)
           if (issued & (1u << st)) drain_wait(&bars[bWfull + st], (last_phase >> st) & 1u);
       }
     }
@@ -205,47 +224,52 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
     if (lane == 0) {
       const uint32_t idz = idesc_bf16_f32(kFR, kFV, false, false);
       const uint32_t ido = idesc_bf16_f32(kFR, a.ds, false, true);
-      const uint32_t ring_a = smem_u32(ring), p_a = smem_u32(ptile);
+      const uint32_t ring_a = smem_u32(ring), p_a = smem_u32(ptiles);
       uint32_t t = 0;
       bool ok = true;
-      // O += P W for tile tt (j-th of sweep s): P K-major (2 atoms of 64 columns),
-      // W slice MN-major (atoms of 64 d-columns kFAtom apart).
+      // O += P W for tile tt (the j-th of sweep s): P K-major (one atom), the W
+      // slice MN-major (atoms of 64 d-columns, kFAtom apart).
       auto issue_o = [&](int j, uint32_t tt, int s) -> bool {
-        if (!mbar_wait_cluster(&bars[bPfull], tt & 1, abort_flag)) return false;
+        const int b = tt & 1;
+        if (!mbar_wait_cluster(&bars[bPfull + b], (tt >> 1) & 1, abort_flag)) return false;
         if (j == 0 && s > 0 && !mbar_wait(&bars[bOempty], (s - 1) & 1, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t sb = ring_a + (tt & 1) * kFStageBytes;
+        const uint32_t sb = ring_a + (tt % kFStages) * kFStageBytes;
+        const uint32_t pb = p_a + b * kFPBytes;
 #pragma unroll
         for (int k = 0; k < kFV / 16; ++k) {
-          const uint64_t ad = smem_desc_sw128(p_a + (k / 4) * kFAtom + (k % 4) * 32, 16, 1024);
+          const uint64_t ad = smem_desc_sw128(pb + k * 32, 16, 1024);
           const uint64_t bd = smem_desc_sw128(sb + k * 2048, kFAtom, 1024);
           mma_bf16(tmem + kTO, ad, bd, ido, (j > 0 || k > 0) ? 1u : 0u);
         }
-        mma_commit_multicast(&bars[bPfree], kAll);   // this CTA's P tile is free again
-        mma_commit(&bars[bWempty + (tt & 1)]);
+        mma_commit_multicast(&bars[bPfree + b], kAll);   // this CTA's P buffer is free again
+        mma_commit(&bars[bWempty + tt % kFStages]);
         return true;
       };
       for (int s = 0; ok; ++s) {
         if (!(ok = mbar_wait(&bars[bXready], s & 1, abort_flag))) break;
         if (!info->valid) break;
         tc_fence_after();
+        const uint32_t t0 = t;
         for (int j = 0; j < a.n_tiles; ++j, ++t) {
-          const int st = t & 1;
-          if (!(ok = mbar_wait(&bars[bWfull + st], (t >> 1) & 1, abort_flag))) break;
-          if (t > 0 && !(ok = mbar_wait(&bars[bZempty], (t - 1) & 1, abort_flag))) break;
+          const int st = t % kFStages, b = t & 1;
+          if (!(ok = mbar_wait(&bars[bWfull + st], (t / kFStages) & 1, abort_flag))) break;
+          if (t >= 2 && !(ok = mbar_wait(&bars[bZempty + b], ((t >> 1) - 1) & 1, abort_flag))) break;
           tc_fence_after();
           const uint32_t sb = ring_a + st * kFStageBytes;
           // partial Z = xhat slice (tensor memory) x W slice^T (K-major atoms)
           for (int k = 0; k < a.ds / 16; ++k) {
             const uint64_t bd = smem_desc_sw128(sb + (k / 4) * kFAtom + (k % 4) * 32, 16, 1024);
-            mma_bf16_ts(tmem + kTZ, tmem + kTX + 8 * k, bd, idz, k > 0 ? 1u : 0u);
+            mma_bf16_ts(tmem + kTZ + b * kFV, tmem + kTX + 8 * k, bd, idz, k > 0 ? 1u : 0u);
           }
-          mma_commit(&bars[bZfull]);
-          // the previous tile's O product while this tile's partial Z is exchanged
-          if (j > 0 && !(ok = issue_o(j - 1, t - 1, s))) break;
+          mma_commit(&bars[bZfull + b]);
+          // the O product of an earlier tile while this tile's partial Z is exchanged
+          if (j >= kFLag && !(ok = issue_o(j - kFLag, t - kFLag, s))) break;
         }
         if (!ok) break;
-        if (!(ok = issue_o(a.n_tiles - 1, t - 1, s))) break;
+        const int first = a.n_tiles > kFLag ? a.n_tiles - kFLag : 0;
+        for (int j = first; ok && j < a.n_tiles; ++j) ok = issue_o(j, t0 + j, s);
+        if (!ok) break;
         mma_commit(&bars[bOfull]);
       }
       if (!ok) {
@@ -262,8 +286,8 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
     const int rr = 32 * q + lane;                      // row within the block
     const int owner = rr / R;
     const int ri = rr - owner * R;
-    const uint32_t part_dst =
-        map_to_rank(smem_u32(part + (static_cast<int>(rank) * R + ri) * kFV * 4), owner);
+    const int prow_src = static_cast<int>(rank) * R + ri;   // row in the owner's buffer
+    const uint32_t part_dst = map_to_rank(smem_u32(parts + prow_src * kFV * 4), owner);
     const uint32_t part_bar = map_to_rank(smem_u32(&bars[bPartFull]), owner);
     const int slice_cols = max(0, min(a.ds, a.d - col0));   // valid d-columns of the slice
     uint32_t t = 0;
@@ -302,38 +326,42 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
       if (!valid) break;
 
       for (int j = 0; j < a.n_tiles; ++j, ++t) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars[bZfull], t & 1, abort_flag) &&
-                                         mbar_wait_cluster(&bars[bPartFree], t & 1, abort_flag));
+        const int b = t & 1;
+        const uint32_t ph = (t >> 1) & 1;
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars[bZfull + b], ph, abort_flag) &&
+                                         mbar_wait_cluster(&bars[bPartFree + b], ph, abort_flag));
         if (!ok) break;
         tc_fence_after();
+        const uint32_t dst = part_dst + b * kFPartBytes;
+        const uint32_t bar = part_bar + b * 8;
 #pragma unroll 1
         for (int c = 0; c < kFV / 32; ++c) {
           float v[32];
-          tmem_ld32(tmem + lanes + kTZ + 32 * c, v);
+          tmem_ld32(tmem + lanes + kTZ + b * kFV + 32 * c, v);
 #pragma unroll
           for (int u = 0; u < 8; ++u)
-            st_async_v4(part_dst + (32 * c + 4 * u) * 4, __float_as_uint(v[4 * u]),
+            st_async_v4(dst + (((8 * c + u) ^ (prow_src & 15)) << 4), __float_as_uint(v[4 * u]),
                         __float_as_uint(v[4 * u + 1]), __float_as_uint(v[4 * u + 2]),
-                        __float_as_uint(v[4 * u + 3]), part_bar);
+                        __float_as_uint(v[4 * u + 3]), bar);
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars[bZempty]);
+        if (lane == 0) mbar_arrive(&bars[bZempty + b]);
       }
       if (!ok) break;
 
       // end of the sweep: O is complete and the owners' per-row factors are in
-      // the first 2 KB of the P tile (16 B per row: a, b, coef, overflow bits)
+      // the first 2 KB of P buffer t & 1 (16 B per row: a, b, coef, overflow bits)
       ok = __all_sync(0xffffffffu, mbar_wait(&bars[bOfull], s & 1, abort_flag) &&
                                        mbar_wait_cluster(&bars[bRfull], s & 1, abort_flag));
       if (!ok) break;
       tc_fence_after();
-      const float4* rf = reinterpret_cast<const float4*>(ptile);
+      const float4* rowfac = reinterpret_cast<const float4*>(ptiles + (t & 1) * kFPBytes);
       uint32_t over = 0;
 #pragma unroll
-      for (int u = 0; u < 4; ++u) over |= __float_as_uint(rf[lane + 32 * u].w);
+      for (int u = 0; u < 4; ++u) over |= __float_as_uint(rowfac[lane + 32 * u].w);
       const bool redo_next = !redo && __any_sync(0xffffffffu, over != 0u);
-      const float4 f = rf[rr];
+      const float4 f = rowfac[rr];
       __syncwarp();
       if (warp == 2 && lane == 0) mbar_arrive_expect_tx(&bars[bRfull], kFR * 16);
       if (!redo_next && slice_cols > 0) {
@@ -366,7 +394,8 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
             const uint4 hv = __ldg(reinterpret_cast<const uint4*>(hrow + col));
             const uint4 gv = __ldg(reinterpret_cast<const uint4*>(a.gamma + col));
             uint4 wv = make_uint4(0, 0, 0, 0);
-            if (use_wy) wv = __ldg(reinterpret_cast<const uint4*>(a.W + static_cast<int64_t>(y) * a.d + col));
+            if (use_wy)
+              wv = __ldg(reinterpret_cast<const uint4*>(a.W + static_cast<int64_t>(y) * a.d + col));
             const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
             const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w};
             const uint32_t ww[4] = {wv.x, wv.y, wv.z, wv.w};
@@ -399,7 +428,6 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
     const int i = ot / TPR;                    // row among this CTA's R rows
     const int g = ot - i * TPR;                // column group of the row
     const int prow = static_cast<int>(rank) * R + i;   // row of the P tile
-    const float* prow_part = reinterpret_cast<const float*>(part) + i * kFV;
     uint32_t t = 0;
     bool ok = true;
     float m_exact = -INFINITY;
@@ -424,31 +452,46 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
       float S = 0.f, U = 0.f, zy = 0.f;
       bool over = false;
       for (int j = 0; j < a.n_tiles; ++j, ++t) {
-        ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPartFull], t & 1, abort_flag));
+        const int b = t & 1;
+        const uint32_t ph = (t >> 1) & 1;
+        ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPartFull + b], ph, abort_flag));
         if (!ok) break;
-        // z = sum of the C partials, in rank order
-        float z[G8][8];
+        // z = sum of the C partials, in rank order.  The row's 64 columns are 16
+        // quads of 4; thread g of the row takes quads g, g + TPR, ...
+        const float* prt = reinterpret_cast<const float*>(parts + b * kFPartBytes);
+        float z[NQ][4];
 #pragma unroll
-        for (int m = 0; m < G8; ++m) {
-          const int cg = g + TPR * m;
+        for (int m = 0; m < NQ; ++m) {
+          const int qd = g + TPR * m;
+          // row src * R + i of the buffer; (src * R + i) & 15 == i & 15 since R >= 16
+          const int pos = 4 * (qd ^ (i & 15));
+          float4 acc = *reinterpret_cast<const float4*>(prt + i * kFV + pos);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) z[m][e] = 0.f;
-#pragma unroll
-          for (int src = 0; src < C; ++src) {
-            const float4* p4 = reinterpret_cast<const float4*>(prow_part + src * R * kFV + 8 * cg);
-            const float4 x0 = p4[0], x1 = p4[1];
-            z[m][0] += x0.x; z[m][1] += x0.y; z[m][2] += x0.z; z[m][3] += x0.w;
-            z[m][4] += x1.x; z[m][5] += x1.y; z[m][6] += x1.z; z[m][7] += x1.w;
+          for (int src = 1; src < C; ++src) {
+            const float4 x = *reinterpret_cast<const float4*>(prt + (src * R + i) * kFV + pos);
+            acc.x += x.x;
+            acc.y += x.y;
+            acc.z += x.z;
+            acc.w += x.w;
           }
+          z[m][0] = acc.x;
+          z[m][1] = acc.y;
+          z[m][2] = acc.z;
+          z[m][3] = acc.w;
         }
+        // the partials are consumed (the loads completed at the barrier): arm the
+        // buffer's next phase and tell every source, one owner thread per source
+        named_bar_and(2, 128, true);
+        if (ot == 0) mbar_arrive_expect_tx(&bars[bPartFull + b], C * R * kFV * 4);
+        if (ot < C) mbar_arrive_remote_relaxed(map_to_rank(smem_u32(&bars[bPartFree + b]), ot));
         const int cbase = j * kFV;
         float tmax = -INFINITY;
 #pragma unroll
-        for (int m = 0; m < G8; ++m) {
-          const int cg = g + TPR * m;
+        for (int m = 0; m < NQ; ++m) {
+          const int qd = g + TPR * m;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            if (cbase + 8 * cg + e >= a.V) z[m][e] = -INFINITY;   // past the vocabulary
+          for (int e = 0; e < 4; ++e) {
+            if (cbase + 4 * qd + e >= a.V) z[m][e] = -INFINITY;   // past the vocabulary
             tmax = fmaxf(tmax, z[m][e]);
           }
         }
@@ -462,62 +505,49 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
         // the target's own term is left out of S, U and P; its logit is kept
         const int yrel = kept ? y - cbase : -1;
 #pragma unroll
-        for (int m = 0; m < G8; ++m) {
-          const int cg = g + TPR * m;
+        for (int m = 0; m < NQ; ++m) {
+          const int qd = g + TPR * m;
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (8 * cg + e == yrel) {
+          for (int e = 0; e < 4; ++e)
+            if (4 * qd + e == yrel) {
               zy = z[m][e];
               z[m][e] = -INFINITY;
             }
         }
-        // the partials are consumed: arm the next phase, tell every source
-        named_bar_and(2, 128, true);
-        if (ot == 0) {
-          mbar_arrive_expect_tx(&bars[bPartFull], C * R * kFV * 4);
-          for (int c = 0; c < C; ++c) mbar_arrive_remote(map_to_rank(smem_u32(&bars[bPartFree]), c));
-        }
-        // every CTA's product of the previous tile is done: the P tiles are free
-        ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPfree], t & 1, abort_flag));
+        // every CTA's product of the buffer's previous tile is done: it is free
+        ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPfree + b], ph, abort_flag));
         if (!ok) break;
+        uint8_t* ptile = ptiles + b * kFPBytes;
         const bool live = kept && !over;
         const float ml = mref * kLog2e;
 #pragma unroll
-        for (int m = 0; m < G8; ++m) {
-          uint32_t pk[4];
+        for (int m = 0; m < NQ; ++m) {
+          float e4[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            float e0 = 0.f, e1 = 0.f;
-            if (live) {
-              e0 = ex2_approx(fmaf(z[m][2 * e], kLog2e, -ml));
-              e1 = ex2_approx(fmaf(z[m][2 * e + 1], kLog2e, -ml));
-            }
-            S += e0 + e1;
-            U += (e0 > 0.f ? e0 * z[m][2 * e] : 0.f) + (e1 > 0.f ? e1 * z[m][2 * e + 1] : 0.f);
-            pk[e] = pack_bf16x2(e0, e1);
+            e4[e] = live ? ex2_approx(fmaf(z[m][e], kLog2e, -ml)) : 0.f;
+            S += e4[e];
+            U += e4[e] > 0.f ? e4[e] * z[m][e] : 0.f;
           }
-          const int cg = g + TPR * m;          // 8-column group: atom cg / 8, chunk cg % 8
-          const uint32_t addr = smem_u32(ptile + (cg >> 3) * kFAtom + prow * 128 +
-                                         (((cg & 7) ^ (prow & 7)) << 4));
-          st_shared_v4(addr, pk[0], pk[1], pk[2], pk[3]);
+          // quad qd = half of the 16-byte chunk qd / 2 of the (swizzled) P row
+          const int qd = g + TPR * m;
+          const uint32_t addr =
+              smem_u32(ptile + prow * 128 + ((((qd >> 1) ^ (prow & 7)) << 4) | ((qd & 1) << 3)));
+          asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr),
+                       "r"(pack_bf16x2(e4[0], e4[1])), "r"(pack_bf16x2(e4[2], e4[3]))
+                       : "memory");
         }
         fence_proxy_async_smem();
         named_bar_and(2, 128, true);
-        if (ot == 0) {
-          // this CTA's R rows of P to every other CTA of the cluster (one copy per atom)
-#pragma unroll 1
-          for (int c = 1; c < C; ++c) {
-            const uint32_t peer = (rank + c) % C;
-            const uint32_t bar = map_to_rank(smem_u32(&bars[bPfull]), peer);
-#pragma unroll
-            for (int at = 0; at < 2; ++at) {
-              const uint32_t off = at * kFAtom + static_cast<int>(rank) * R * 128;
-              bulk_copy_s2s(map_to_rank(smem_u32(ptile + off), peer), smem_u32(ptile + off),
-                            R * 128, bar);
-            }
-          }
-          mbar_arrive_expect_tx(&bars[bPfull], (C - 1) * R * 256);
+        // this CTA's R rows of P to every other CTA of the cluster, one owner
+        // thread per peer
+        if (ot < C - 1) {
+          const uint32_t off = b * kFPBytes + static_cast<int>(rank) * R * 128;
+          const uint32_t peer = (rank + 1 + ot) % C;
+          bulk_copy_s2s(map_to_rank(smem_u32(ptiles + off), peer), smem_u32(ptiles + off),
+                        R * 128, map_to_rank(smem_u32(&bars[bPfull + b]), peer));
         }
+        if (ot == C - 1) mbar_arrive_expect_tx(&bars[bPfull + b], (C - 1) * R * 128);
       }
       if (!ok) break;
       // ---- end of the sweep: the row's totals over its TPR threads
@@ -545,16 +575,18 @@ __global__ void __cluster_dims__(C, 1, 1) __launch_bounds__(kFThreads, 1)
         if (a.loss_tok) a.loss_tok[row] = loss;
         a.row_loss[row] = loss;
       }
-      // every CTA's last product of the sweep is done: its P tile can hold the factors
-      ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPfree], t & 1, abort_flag));
+      // P buffer t & 1 (its last user, tile t - 2, is done everywhere) carries the
+      // factors; the next sweep's owners write it only after every CTA's lanes
+      // have read them (their partials of that sweep come after)
+      ok = named_bar_and(1, 128, mbar_wait_cluster(&bars[bPfree + (t & 1)], (t >> 1) & 1, abort_flag));
       if (!ok) break;
       if (g == 0) {
         const uint32_t ob = over ? 1u : 0u;
+        const uint32_t dst = smem_u32(ptiles + (t & 1) * kFPBytes + prow * 16);
 #pragma unroll 1
         for (int c = 0; c < C; ++c)
-          st_async_v4(map_to_rank(smem_u32(ptile + prow * 16), c), __float_as_uint(fa),
-                      __float_as_uint(fb), __float_as_uint(fcoef), ob,
-                      map_to_rank(smem_u32(&bars[bRfull]), c));
+          st_async_v4(map_to_rank(dst, c), __float_as_uint(fa), __float_as_uint(fb),
+                      __float_as_uint(fcoef), ob, map_to_rank(smem_u32(&bars[bRfull]), c));
       }
     }
     if (!ok && ot == 0) atomicOr(a.flags, SOLO_FLAG_TIMEOUT);

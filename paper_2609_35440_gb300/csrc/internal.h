@@ -163,7 +163,7 @@ struct FlashArgs {
   int32_t d;
   int32_t V;
   int32_t ds;            // d-columns per CTA (multiple of 64, <= 256)
-  int32_t n_tiles;       // 128-column vocabulary tiles
+  int32_t n_tiles;       // 64-column vocabulary tiles
   int32_t row_blocks;    // 128-row blocks
   int64_t N;             // tokens per module
   int32_t modules;       // auxiliary modules (K - 1)
@@ -193,7 +193,7 @@ cudaError_t flash_prepare(int device);
 // Kept-token counts and 1/Nvalid of the auxiliary modules (and bad-target flags).
 cudaError_t launch_flash_count(const FlashArgs& a, float* inv_nvalid, cudaStream_t s);
 // The on-chip forward + backward of the auxiliary rows; w: tensor map of W
-// (bf16 [V, d], 64 x 128 boxes, 128-byte swizzle).
+// (bf16 [V, d], boxes of 64 columns x 64 rows, 128-byte swizzle).
 cudaError_t launch_flash(const CUtensorMap& w, const FlashArgs& a, int device, int sms,
                          cudaStream_t s);
 // Module means of the auxiliary modules from row_loss, in a fixed order.

@@ -694,7 +694,7 @@ solo_status_t run_onchip(const solo_dims_t* dims, const solo_bf16_t* const* hidd
   fa.d = D.d;
   fa.V = D.V;
   fa.ds = flash_slice_width(D.d);
-  fa.n_tiles = (D.V + 127) / 128;
+  fa.n_tiles = (D.V + 63) / 64;
   fa.row_blocks = static_cast<int32_t>((static_cast<int64_t>(fa.M) + 127) / 128);
   fa.N = D.N;
   fa.modules = aux;
@@ -735,7 +735,7 @@ solo_status_t run_onchip(const solo_dims_t* dims, const solo_bf16_t* const* hidd
         launch_flash_count(fa, inv_nvalid, stream) != cudaSuccess)
       return SOLO_ERR_CUDA;
     if (!make_map(&mW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, W, static_cast<uint64_t>(D.d),
-                  static_cast<uint64_t>(D.V), static_cast<uint64_t>(D.d) * 2, 64, 128))
+                  static_cast<uint64_t>(D.V), static_cast<uint64_t>(D.d) * 2, 64, 64))
       return SOLO_ERR_CUDA;
   }
   if (!mark(SOLO_ONCHIP_STAGE_AUX)) return SOLO_ERR_CUDA;
