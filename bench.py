@@ -137,9 +137,10 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def committed_traffic(wl):
+def committed_traffic(wl, kept_tokens: int):
     """Bytes per launch of the logits GEMM from the committed ncu capture, if the
-    kernel source is unchanged since; scaled by the tiles of this workload."""
+    kernel source is unchanged since; scaled to this workload's kept tokens x
+    vocabulary tiles (the reads also by d)."""
     try:
         kv = {}
         with open(TRAFFIC_FILE) as f:
@@ -149,8 +150,9 @@ def committed_traffic(wl):
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_sha") != kernel_hash():
             return None
-        per_unit = float(kv["dram_bytes_per_token_per_vocab_tile"])
-        return per_unit * wl.M * ((wl.V + 255) // 256) * (wl.d / float(kv["d"]))
+        w = float(kv["dram_write_bytes_per_token_per_vocab_tile"])
+        r = float(kv["dram_read_bytes_per_token_per_vocab_tile"])
+        return kept_tokens * ((wl.V + 255) // 256) * (w + r * wl.d / float(kv["d"]))
     except (OSError, KeyError, ValueError):
         return None
 
@@ -511,6 +513,8 @@ def run_ours(args, wl):
 
     peaks, peak_src = load_peaks()
     G = costmodel.gemm_flops(wl.M, wl.V, wl.d)     # one module-GEMM over all K modules
+    n_kept = kept_counts(wl, inp.targets)
+    Gk = costmodel.gemm_flops(sum(n_kept), wl.V, wl.d)   # over the kept tokens
     if onchip:
         names = sr.ONCHIP_STAGE_NAMES
         # final module: logits, dX and dW over its N tokens; auxiliary modules: the
@@ -518,14 +522,17 @@ def run_ours(args, wl):
         gemm_stage_flops = {"final": 3 * G / wl.K, "aux_onchip": 2 * G * (wl.K - 1) / wl.K}
     else:
         names = sr.STAGE_NAMES
-        gemm_stage_flops = {"logits": G, "dxhat": G, "dW": G / wl.K}
+        # masked tokens are skipped: the logits and dX products run over the kept
+        # tokens; dW reduces over the final module's N rows (kept ones, then zeros)
+        gemm_stage_flops = {"logits": Gk, "dxhat": Gk, "dW": G / wl.K}
     dom = max(gemm_stage_flops, key=lambda s: stage_ms[names.index(s)])
     dom_ms = stage_ms[names.index(dom)]
     achieved = gemm_stage_flops[dom] / (dom_ms / 1e3) / 1e12
     peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
-    traffic = committed_traffic(wl) if dom == "logits" and not onchip else None
+    traffic = committed_traffic(wl, sum(n_kept)) if dom == "logits" and not onchip else None
     algo = costmodel.call_flops(wl.K, wl.N, wl.d, wl.V)
-    kept = costmodel.kept_call_flops(kept_counts(wl, inp.targets), wl.d, wl.V)
+    kept = costmodel.kept_call_flops(n_kept, wl.d, wl.V)
+    executed = sum(gemm_stage_flops.values())
     step_s = ms / 1e3 / args.steps
     cpu = None
     if not args.no_cpu:
@@ -547,9 +554,9 @@ def run_ours(args, wl):
         # every product; the mean loss counts kept tokens)
         "kept_algo_tflops": kept / step_s / 1e12,
         "kept_algo_frac_of_peak": kept / step_s / 1e12 / peak,
-        # the tensor cores execute exactly the algorithmic (2K+1) 2NVd: no logits
-        # are recomputed (the forward stores its exponentials)
-        "executed_tflops": algo / step_s / 1e12,
+        # what the tensor cores execute: no logits are recomputed (the forward
+        # stores its exponentials) and masked tokens are skipped
+        "executed_tflops": executed / step_s / 1e12,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
         "roofline": {"bound": "tensor",
                      "kernel": ("auxiliary on-chip pass (tcgen05, cluster split of d)"

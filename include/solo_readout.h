@@ -124,6 +124,10 @@ solo_status_t solo_readout_workspace_bytes(const solo_dims_t* dims, size_t* byte
  *             marks masked tokens; anything else outside [0, V) is treated
  *             as masked and sets SOLO_FLAG_BAD_TARGET.
  *  mask       uint8 [K, N] or NULL: 0 masks the token (ANDed with the above).
+ *             Masked tokens are skipped by every product: the kept ones are
+ *             compacted (in token order) into the first rows of the workspace's
+ *             per-token buffers, so the call's tensor work scales with the kept
+ *             tokens.
  *  loss_tok   fp32 [K, N] or NULL: per-token cross-entropy, 0 when masked.
  *  loss_mean  fp32 [K]: L_k, mean over kept tokens (0 when none is kept).
  *  dhidden    host array [K] of device pointers, each bf16 [N, d]:
@@ -448,7 +452,7 @@ uint64_t solo_readout_kernel_launches(void);
  *  - Problems whose solo_readout_workspace_bytes exceeds
  *    SOLO_STATIC_SCRATCH_BYTES are rejected with
  *    SOLO_ERR_EXCEEDS_STATIC_SCRATCH before anything is enqueued (roughly
- *    K*N*(2.0625*V + 2*d + 24) bytes plus up to 32 MiB of partial tiles of the
+ *    K*N*(2.0625*V + 2*d + 36) bytes plus up to 32 MiB of partial tiles of the
  *    backward products must fit; e.g. K=2, N=256, d=128, V=4096 uses about
  *    8.3 MiB).
  *  - The first call on a device looks up the device address of the scratch

@@ -77,11 +77,41 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 constexpr uint16_t kBothCtas = 0x3;
 
-__device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, int& nb) {
+// The product's rows and its work units.  From the host's GemmArgs, or, with
+// compacted rows (m_dev), planned here from the device row count with the
+// host's rule (plan_units): whole tiles fill complete waves of pairs, the rest
+// is cut along the reduction.
+struct Plan {
+  int M, m_blocks, num_tiles, full_tiles, split, num_units;
+};
+
+__device__ __forceinline__ Plan make_plan(const GemmArgs& a) {
+  Plan p{a.M, a.m_blocks, a.num_tiles, a.full_tiles, a.split, a.num_units};
+  if (a.m_dev == nullptr) return p;
+  p.M = min(*a.m_dev, a.M);
+  p.m_blocks = (p.M + 2 * kBM - 1) / (2 * kBM);
+  p.num_tiles = p.m_blocks * a.n_blocks;
+  p.full_tiles = p.num_tiles;
+  p.split = 1;
+  p.num_units = p.num_tiles;
+  const int pairs = min(max(a.sms / 2, 1), kMaxAuxSlots + 1);
+  const int rem = p.num_tiles % pairs;
+  if (!a.split_ok || rem == 0) return p;
+  int s = min(min(pairs / rem, kMaxSplit), a.k_blocks);
+  while (s > 1 && rem * (a.aux_part0 ? s : s - 1) > min(a.aux_slots, kMaxAuxSlots)) --s;
+  if (s < 2) return p;
+  p.full_tiles = p.num_tiles - rem;
+  p.split = s;
+  p.num_units = p.full_tiles + rem * s;
+  return p;
+}
+
+__device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, const Plan& p, int& mb,
+                                            int& nb) {
   const int per_group = a.group_m * a.n_blocks;
   const int g = t / per_group;
   const int first_m = g * a.group_m;
-  const int gm = min(a.m_blocks - first_m, a.group_m);
+  const int gm = min(p.m_blocks - first_m, a.group_m);
   const int r = t - g * per_group;
   mb = first_m + r % gm;
   nb = r / gm;
@@ -89,20 +119,20 @@ __device__ __forceinline__ void tile_coords(int t, const GemmArgs& a, int& mb, i
 
 // Work unit u -> tile, part of the tile (0 for a whole tile) and its
 // reduction blocks [kb_lo, kb_hi).
-__device__ __forceinline__ void unit_range(int u, const GemmArgs& a, int& t, int& part,
-                                           int& kb_lo, int& kb_hi) {
-  if (u < a.full_tiles) {
+__device__ __forceinline__ void unit_range(int u, const GemmArgs& a, const Plan& p, int& t,
+                                           int& part, int& kb_lo, int& kb_hi) {
+  if (u < p.full_tiles) {
     t = u;
     part = 0;
     kb_lo = 0;
     kb_hi = a.k_blocks;
     return;
   }
-  const int i = u - a.full_tiles;
-  t = a.full_tiles + i / a.split;
-  part = i % a.split;
-  kb_lo = static_cast<int>(static_cast<int64_t>(part) * a.k_blocks / a.split);
-  kb_hi = static_cast<int>(static_cast<int64_t>(part + 1) * a.k_blocks / a.split);
+  const int i = u - p.full_tiles;
+  t = p.full_tiles + i / p.split;
+  part = i % p.split;
+  kb_lo = static_cast<int>(static_cast<int64_t>(part) * a.k_blocks / p.split);
+  kb_hi = static_cast<int>(static_cast<int64_t>(part + 1) * a.k_blocks / p.split);
 }
 
 // Waits without looking at the abort flag, bounded in time: used to drain
@@ -143,16 +173,19 @@ struct NormRow {
   uint16_t* dh;        // the row of dhidden (bf16)
 };
 
-__device__ __forceinline__ NormRow norm_row(const GemmArgs& g, int64_t row) {
+// dg_row0: first row of the final module (compacted rows: its first kept token).
+__device__ __forceinline__ NormRow norm_row(const GemmArgs& g, int64_t row, int M,
+                                            int64_t dg_row0) {
   NormRow nr{false, false, 0.f, 0.f, nullptr, nullptr};
-  if (row >= g.M) return nr;
-  const int k = static_cast<int>(row / g.tokens_per_module);
+  if (row >= M) return nr;
+  const int64_t tok = g.orig_row ? g.orig_row[row] : row;
+  const int k = static_cast<int>(tok / g.tokens_per_module);
   if (!in_bounds(k < g.modules, g.flags)) return nr;
-  const int64_t n = row - static_cast<int64_t>(k) * g.tokens_per_module;
+  const int64_t n = tok - static_cast<int64_t>(k) * g.tokens_per_module;
   const float r = g.r[row];
   const float tau = g.tau ? g.tau[k] : 1.f;
   nr.ok = true;
-  nr.dg = g.dg_part != nullptr && row >= g.dg_row0;
+  nr.dg = g.dg_part != nullptr && row >= dg_row0;
   nr.r = r;
   nr.coef = r * r * (tau * g.inv_nvalid[k] * g.edz[row]) / static_cast<float>(g.N);
   nr.h = g.hidden[k] + n * g.N;
@@ -232,8 +265,9 @@ __device__ __forceinline__ void norm_bwd_chunk(const GemmArgs& g, const float (&
 // The dgamma partial row of the 32-row block starting at row_base (a multiple
 // of 32), for columns from col0.  Callers ask only for blocks holding a row of
 // the final module; a checked build tests that and returns null otherwise.
-__device__ __forceinline__ float* dg_block(const GemmArgs& g, int64_t row_base, int col0) {
-  const int64_t rb = (row_base >> 5) - (g.dg_row0 >> 5);
+__device__ __forceinline__ float* dg_block(const GemmArgs& g, int64_t row_base, int col0,
+                                           int64_t dg_row0) {
+  const int64_t rb = (row_base >> 5) - (dg_row0 >> 5);
   if (g.dg_part == nullptr || !in_bounds(rb >= 0 && rb < g.dg_blocks, g.flags)) return nullptr;
   return g.dg_part + rb * g.N + col0;
 }
@@ -270,6 +304,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   const bool even = rank == 0;
   const int cluster = blockIdx.x >> 1;
   const int num_clusters = gridDim.x >> 1;
+  const Plan plan = make_plan(args);
+  // kDW: first reduction row (the final module's first token); kDxhat: first
+  // row of the final module, for the dgamma blocks; read from device memory
+  // when the rows are compacted
+  const int64_t dev_row0 = args.row0_dev ? static_cast<int64_t>(*args.row0_dev) : -1;
+  const int64_t kred0 = (MODE == kDW && dev_row0 >= 0) ? dev_row0 : args.k_row0;
+  const int64_t row0 = (MODE == kDxhat && dev_row0 >= 0) ? dev_row0 : args.dg_row0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -304,10 +345,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       uint32_t stage = 0, phase = 0;
       uint32_t issued = 0, last_phase = 0;   // per-stage bits for draining
       bool ok = true;
-      for (int u = cluster; ok && u < args.num_units; u += num_clusters) {
+      for (int u = cluster; ok && u < plan.num_units; u += num_clusters) {
         int t, part, kb_lo, kb_hi, mb, nb;
-        unit_range(u, args, t, part, kb_lo, kb_hi);
-        tile_coords(t, args, mb, nb);
+        unit_range(u, args, plan, t, part, kb_lo, kb_hi);
+        tile_coords(t, args, plan, mb, nb);
         const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
         const int n0 = nb * kBN + static_cast<int>(rank) * kBHalf;
         for (int kb = kb_lo; kb < kb_hi; ++kb) {
@@ -319,7 +360,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           uint8_t* sB = smem + kSmemB + stage * kBBytes;
           if (even) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
           const uint32_t fb = full_even + stage * 8;
-          const int kr = args.k_row0 + kb * kBK;
+          const int kr = static_cast<int>(kred0) + kb * kBK;
           if constexpr (!kAmn) {
 #pragma unroll
             for (int a = 0; a < kKAtoms; ++a)
@@ -377,9 +418,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       bool ok = true;
       const uint32_t a_base = smem_u32(smem + kSmemA);
       const uint32_t b_base = smem_u32(smem + kSmemB);
-      for (int u = cluster; ok && u < args.num_units; u += num_clusters, ++local) {
+      for (int u = cluster; ok && u < plan.num_units; u += num_clusters, ++local) {
         int t, part, kb_lo, kb_hi;
-        unit_range(u, args, t, part, kb_lo, kb_hi);
+        unit_range(u, args, plan, t, part, kb_lo, kb_hi);
         const uint32_t acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait_cluster(&tempty[acc], acc_phase ^ 1, abort_flag)) {
@@ -433,10 +474,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     int buf = 0;
     int local = 0;
     bool ok = true;
-    for (int u = cluster; u < args.num_units; u += num_clusters, ++local) {
+    for (int u = cluster; u < plan.num_units; u += num_clusters, ++local) {
       int t, part, kb_lo, kb_hi, mb, nb;
-      unit_range(u, args, t, part, kb_lo, kb_hi);
-      tile_coords(t, args, mb, nb);
+      unit_range(u, args, plan, t, part, kb_lo, kb_hi);
+      tile_coords(t, args, plan, mb, nb);
       const int m0 = mb * kPairRows + static_cast<int>(rank) * kBM;
       const int n0 = nb * kBN;
       const uint32_t acc = local & 1;
@@ -449,7 +490,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const int ncols = min(kBN, args.N - n0);    // valid columns, warp-uniform
 
       if constexpr (MODE == kExit) {
-        const bool row_ok = row < args.M;
+        const bool row_ok = row < plan.M;
         const int y = (row_ok && args.targets) ? args.targets[row] : -1;
         const int yrel = y - n0;
         const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
@@ -512,7 +553,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         if (has_y) args.zy[row] = zyv;
       } else if constexpr (MODE == kLogits || MODE == kLogitsHeads) {
         constexpr bool kHeads = (MODE == kLogitsHeads);
-        const bool row_ok = row < args.M;
+        const bool row_ok = row < plan.M;
         const int y = row_ok ? args.targets[row] : -1;
         const int yrel = y - n0;
         const bool has_y = row_ok && y >= 0 && y < args.V && yrel >= 0 && yrel < ncols;
@@ -520,7 +561,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         float tau = 1.f;
         const float* brow = nullptr;
         if constexpr (kHeads) {
-          const int kmod = row_ok ? static_cast<int>(row / args.tokens_per_module) : 0;
+          const int64_t tok = row_ok ? (args.orig_row ? args.orig_row[row] : row) : 0;
+          const int kmod = static_cast<int>(tok / args.tokens_per_module);
           if (args.tau) tau = args.tau[kmod];
           if (args.bias &&
               in_bounds(kmod < args.M / args.tokens_per_module && n0 + ncols <= args.V,
@@ -672,11 +714,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           if (has_y) args.sy[row] = syv;
         }
         if (has_y) args.zy[row] = zyv;
-      } else if (MODE == kDxhat && args.norm_fused && t < args.full_tiles) {
+      } else if (MODE == kDxhat && args.norm_fused && t < plan.full_tiles) {
         // whole dX̂ tile: the RMSNorm backward straight from TMEM to bf16 dH
-        const NormRow nr = norm_row(args, row);
+        const NormRow nr = norm_row(args, row, plan.M, row0);
         const bool dg_warp = __any_sync(0xffffffffu, nr.dg);
-        float* dg = dg_warp ? dg_block(args, m0 + 32 * q, n0) : nullptr;
+        float* dg = dg_warp ? dg_block(args, m0 + 32 * q, n0, row0) : nullptr;
         for (int c = 0; c < kBN / 32; ++c) {
           if (c * 32 >= ncols) break;
           float v[32];
@@ -711,9 +753,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             if (part == 0 && !args.aux_part0) {
               tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + c * 32, m0 + 32 * q);
             } else {    // a reduction range of a cut tile: its auxiliary slot
-              const int cut = t - args.full_tiles;
-              const int slot = args.aux_part0 ? cut * args.split + part
-                                              : cut * (args.split - 1) + part - 1;
+              const int cut = t - plan.full_tiles;
+              const int slot = args.aux_part0 ? cut * plan.split + part
+                                              : cut * (plan.split - 1) + part - 1;
               if (in_bounds(slot >= 0 && slot < args.aux_slots, args.flags))
                 tma_store_2d(&tmX, ebuf + buf * kEpiBufBytes, c * 32,
                              slot * kPairRows + static_cast<int>(rank) * kBM + 32 * q);
@@ -764,6 +806,8 @@ cudaError_t gemm_prepare(int /*device*/) {
 }
 
 void plan_units(GemmArgs& g, int sms, bool allow_split) {
+  g.sms = sms;
+  g.split_ok = allow_split ? 1 : 0;
   g.full_tiles = g.num_tiles;
   g.split = 1;
   g.num_units = g.num_tiles;
@@ -784,21 +828,23 @@ namespace {
 // Grid (cut tiles, 256 / 16 row chunks), 256 threads: 16 rows x 64 float4.
 __global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, float* out,
                                                           int64_t ld, const float* aux) {
+  const Plan plan = make_plan(g);
   const int cut = blockIdx.x;
-  const int t = g.full_tiles + cut;
+  if (cut >= plan.num_tiles - plan.full_tiles) return;
+  const int t = plan.full_tiles + cut;
   int mb, nb;
-  tile_coords(t, g, mb, nb);
+  tile_coords(t, g, plan, mb, nb);
   const int lr = blockIdx.y * 16 + (threadIdx.x >> 6);     // row within the tile (+ 4 x 4)
   const int c4 = threadIdx.x & 63;                          // float4 column within the tile
   const int col = nb * kBN + 4 * c4;
   for (int rr = 0; rr < 16; rr += 4) {
     const int r = lr + rr;
     const int64_t row = static_cast<int64_t>(mb) * kPairRows + r;
-    if (row >= g.M || col >= g.N) continue;        // N is a multiple of 8: whole float4s
+    if (row >= plan.M || col >= g.N) continue;     // N is a multiple of 8: whole float4s
     float4* o = reinterpret_cast<float4*>(out + row * ld + col);
     float4 acc = *o;
-    for (int p = 1; p < g.split; ++p) {
-      const int slot = cut * (g.split - 1) + p - 1;
+    for (int p = 1; p < plan.split; ++p) {
+      const int slot = cut * (plan.split - 1) + p - 1;
       if (!in_bounds(slot < g.aux_slots, g.flags)) continue;
       const float4 x = *reinterpret_cast<const float4*>(
           aux + (static_cast<int64_t>(slot) * kPairRows + r) * kBN + 4 * c4);
@@ -816,10 +862,13 @@ __global__ void __launch_bounds__(256) split_fixup_kernel(const GemmArgs g, floa
 // the order split_fixup_kernel adds them in).  Grid (cut tiles, 8 blocks of 32
 // rows); warp w handles the tile's columns [32 w, 32 w + 32), lane i row i.
 __global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, const float* aux) {
+  const Plan plan = make_plan(g);
   const int cut = static_cast<int>(blockIdx.x);
-  const int t = g.full_tiles + cut;
+  if (cut >= plan.num_tiles - plan.full_tiles) return;   // (launched for the most cut tiles)
+  const int t = plan.full_tiles + cut;
   int mb, nb;
-  tile_coords(t, g, mb, nb);
+  tile_coords(t, g, plan, mb, nb);
+  const int64_t row0 = g.row0_dev ? static_cast<int64_t>(*g.row0_dev) : g.dg_row0;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int lr = blockIdx.y * 32 + lane;                    // row within the tile
@@ -828,13 +877,13 @@ __global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, c
   const int col0 = nb * kBN + warp * 32;
   if (col0 >= g.N) return;                       // warp-uniform
   const int cols = min(32, g.N - col0);
-  const NormRow nr = norm_row(g, row);
+  const NormRow nr = norm_row(g, row, plan.M, row0);
   float v[32];
 #pragma unroll
   for (int j = 0; j < 32; ++j) v[j] = 0.f;
   if (nr.ok) {
-    for (int p = 0; p < g.split; ++p) {
-      const int slot = cut * g.split + p;
+    for (int p = 0; p < plan.split; ++p) {
+      const int slot = cut * plan.split + p;
       if (!in_bounds(slot < g.aux_slots, g.flags)) continue;
       const float4* src = reinterpret_cast<const float4*>(
           aux + (static_cast<int64_t>(slot) * kPairRows + lr) * kBN + warp * 32);
@@ -858,14 +907,17 @@ __global__ void __launch_bounds__(256) cut_tiles_norm_kernel(const GemmArgs g, c
     }
   }
   const bool dg_warp = __any_sync(0xffffffffu, nr.dg);
-  norm_bwd_chunk(g, v, col0, cols, nr, dg_warp, dg_warp ? dg_block(g, row_base, col0) : nullptr);
+  norm_bwd_chunk(g, v, col0, cols, nr, dg_warp,
+                 dg_warp ? dg_block(g, row_base, col0, row0) : nullptr);
 }
 
 }  // namespace
 
 cudaError_t launch_cut_tiles_norm(const GemmArgs& g, const float* aux, cudaStream_t stream) {
-  const int cut = g.num_tiles - g.full_tiles;
-  if (!g.norm_fused || !g.aux_part0 || g.split < 2 || cut <= 0) return cudaSuccess;
+  // compacted rows: the device plans the cut tiles; launch for the most there can be
+  const int pairs = std::min(std::max(g.sms / 2, 1), kMaxAuxSlots + 1);
+  const int cut = g.m_dev ? std::min(pairs - 1, g.num_tiles) : g.num_tiles - g.full_tiles;
+  if (!g.norm_fused || !g.aux_part0 || cut <= 0 || (!g.m_dev && g.split < 2)) return cudaSuccess;
   cut_tiles_norm_kernel<<<dim3(cut, kPairRows / 32), 256, 0, stream>>>(g, aux);
   return launched();
 }

@@ -118,6 +118,16 @@ struct GemmArgs {
   float* dg_part;          // [dg_blocks, d] or null: per 32-row block of the final module
   int32_t dg_blocks;
   int64_t dg_row0;         // first row of the final module
+  // Compacted rows (masked tokens skipped): the row count, the final module's
+  // first row and the token of each row live in device memory.  With m_dev the
+  // kernel plans its tiles and cut tiles itself from *m_dev <= M (the host's
+  // full_tiles / split / num_units describe the upper bound M).
+  const int32_t* m_dev;     // rows of the product, or null (M)
+  const int32_t* row0_dev;  // kDW: first reduction row / kDxhat: first row of the final
+                            //   module (dgamma blocks), or null (k_row0 / dg_row0)
+  const int32_t* orig_row;  // [M]: token (k * N + n) of a row, or null (the row itself)
+  int32_t sms;              // multiprocessors, for the device-side plan
+  int32_t split_ok;         // the plan may cut the last partial wave
 };
 
 size_t gemm_smem_bytes();
@@ -248,10 +258,24 @@ struct RowArgs {
   float* dbias;          // [K, V] or null
   float* db_part;        // [K, db_chunks, ldp]
   int32_t db_chunks;     // row chunks per module of the gradient pass
+  // Compaction of the kept tokens (null kept_local: every token keeps its row).
+  // Kept tokens take rows [0, Mk) of the per-row buffers in token order, module
+  // by module; each masked token zeroes one row of [Mk, M).
+  int32_t* kept_local;   // [M] kept tokens before this one within its chunk of kScanRows
+  int32_t* chunk_base;   // [K * nchunks] kept tokens before the chunk (counts, then prefix)
+  int32_t nchunks;       // chunks of kScanRows tokens per module
+  int32_t* offsets;      // [K + 1] first compact row of each module; offsets[K] = Mk
+  int32_t* orig_row;     // [M] compact row -> token row k * N + n
+  int32_t* tgt_c;        // [M] target of a compact row
 };
+
+constexpr int kScanRows = 1024;  // tokens per block of the kept-token scan
 
 constexpr int kGradRows = 256;   // rows per CTA of the gradient pass
 
+// Kept-token scan (with a.kept_local): per-chunk counts and in-chunk ranks,
+// then the prefix over chunks and the modules' compact offsets.
+cudaError_t launch_keep_scan(const RowArgs& a, cudaStream_t s);
 cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s);
 // heads: with the heads' temperature gradient (a.dtau) as well
 cudaError_t launch_lse(const RowArgs& a, cudaStream_t s, bool heads = false);

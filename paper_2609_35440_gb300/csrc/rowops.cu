@@ -33,6 +33,89 @@ __device__ __forceinline__ bool token_kept(const RowArgs& a, int64_t row, int y)
   return in_range && y != a.ignore_index && (a.mask == nullptr || a.mask[row] != 0);
 }
 
+// ---- kept-token compaction ------------------------------------------------------
+// Masked tokens need no logits and no gradient: the kept ones take rows
+// [0, Mk) of every per-row buffer (token order, module by module), so the
+// products run over Mk rows only.  Ranks are exact integer prefix sums: the
+// compact order is the token order, whatever the schedule.
+
+// Per chunk of kScanRows tokens of module blockIdx.y: each token's count of kept
+// tokens before it within the chunk, and the chunk's total; bad targets flagged.
+__global__ void __launch_bounds__(kScanRows) keep_scan_kernel(const RowArgs a) {
+  __shared__ int warp_tot[kScanRows / 32];
+  const int k = blockIdx.y;
+  const int64_t n = static_cast<int64_t>(blockIdx.x) * kScanRows + threadIdx.x;
+  const int64_t row = static_cast<int64_t>(k) * a.N + n;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int kept = 0, bad = 0;
+  if (n < a.N) {
+    const int y = a.targets[row];
+    kept = token_kept(a, row, y) ? 1 : 0;
+    bad = (!(y >= 0 && y < a.V) && y != a.ignore_index) ? 1 : 0;
+  }
+  const uint32_t ballot = __ballot_sync(0xffffffffu, kept);
+  const int in_warp = __popc(ballot & ((1u << lane) - 1u));
+  if (lane == 0) warp_tot[warp] = __popc(ballot);
+  if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(a.flags, SOLO_FLAG_BAD_TARGET);
+  if (warp == 0) {
+    const int v = warp_tot[lane];          // kScanRows / 32 == 32 warps
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int x = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += x;
+    }
+    warp_tot[lane] = incl - v;             // exclusive prefix of the warp totals
+    if (lane == 31) a.chunk_base[static_cast<int64_t>(k) * a.nchunks + blockIdx.x] = incl;
+  }
+  __syncthreads();
+  if (n < a.N) a.kept_local[row] = warp_tot[warp] + in_warp;
+}
+
+// One block: chunk counts -> exclusive prefix over (module, chunk) in order;
+// offsets[k] = first compact row of module k, offsets[K] = Mk.
+__global__ void __launch_bounds__(1024) keep_offsets_kernel(const RowArgs a) {
+  __shared__ int warp_sum[32];
+  __shared__ int carry_s;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t total = static_cast<int64_t>(a.K) * a.nchunks;
+  if (threadIdx.x == 0) carry_s = 0;
+  __syncthreads();
+  for (int64_t base = 0; base < total; base += 1024) {
+    const int64_t i = base + threadIdx.x;
+    const int v = i < total ? a.chunk_base[i] : 0;
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int x = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += x;
+    }
+    if (lane == 31) warp_sum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const int w = warp_sum[lane];
+      int wi = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, wi, o);
+        if (lane >= o) wi += x;
+      }
+      warp_sum[lane] = wi - w;
+    }
+    __syncthreads();
+    const int carry = carry_s;
+    if (i < total) {
+      const int ex = carry + warp_sum[warp] + incl - v;
+      a.chunk_base[i] = ex;
+      if (i % a.nchunks == 0) a.offsets[i / a.nchunks] = ex;
+    }
+    __syncthreads();
+    if (threadIdx.x == 1023) carry_s = carry + warp_sum[warp] + incl;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) a.offsets[a.K] = carry_s;
+}
+
 // ---- final RMSNorm: r_i = (mean_j h_ij^2 + eps)^-1/2, xhat = bf16(gamma h r) ------
 // The bf16 rounding of xhat is a quantisation decision, so it is taken on the
 // exact value, in fp32 arithmetic only (fp64 is slow on this part):
@@ -131,6 +214,31 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const uint4* h = reinterpret_cast<const uint4*>(a.hidden[k] + n * a.d);
   const uint4* g = reinterpret_cast<const uint4*>(a.gamma);
   const int nv = a.d / 8;
+  int64_t out_row = row;
+  if (a.kept_local != nullptr) {
+    // compact row: kept tokens before this one
+    const int64_t before = a.chunk_base[static_cast<int64_t>(k) * a.nchunks + n / kScanRows] +
+                           a.kept_local[row];
+    const int y = a.targets[row];
+    if (!token_kept(a, row, y)) {
+      // masked: its loss and dH row are zero, and it zeroes one row of [Mk, M)
+      // (the rows past the kept ones that the products read in their last tiles)
+      const int64_t slot = a.offsets[a.K] + (row - before);
+      uint4* xz = reinterpret_cast<uint4*>(a.xhat + slot * a.d);
+      uint4* dz = a.dhidden[k] ? reinterpret_cast<uint4*>(a.dhidden[k] + n * a.d) : nullptr;
+      for (int v = lane; v < nv; v += 32) {
+        if (in_bounds(slot < M, a.flags)) xz[v] = make_uint4(0, 0, 0, 0);
+        if (dz) dz[v] = make_uint4(0, 0, 0, 0);
+      }
+      if (lane == 0 && a.loss_tok) a.loss_tok[row] = 0.f;
+      return;
+    }
+    out_row = before;
+    if (lane == 0 && in_bounds(before < M, a.flags)) {
+      a.orig_row[before] = static_cast<int32_t>(row);
+      a.tgt_c[before] = y;
+    }
+  }
   constexpr int kCache = VPL > 0 ? VPL : 1;
   uint4 hc[kCache];
   // eight independent error-free sums (one per element position of a vector)
@@ -176,7 +284,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   const F2 x = add_f2(F2{m_hi, m_lo}, F2{a.eps, 0.f});
   const F2 rr = rsqrt_f2(x);
   const float r = rr.hi;
-  uint4* out = reinterpret_cast<uint4*>(a.xhat + row * a.d);
+  uint4* out = reinterpret_cast<uint4*>(a.xhat + out_row * a.d);
   auto emit = [&](int v, const uint4& x) {
     float f[8], gg[8];
     unpack8(x, f);
@@ -196,7 +304,7 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
   } else {
     for (int v = lane; v < nv; v += 32) emit(v, __ldg(h + v));
   }
-  if (lane == 0 && a.r) a.r[row] = r;
+  if (lane == 0 && a.r) a.r[out_row] = r;
 }
 
 // ---- log-sum-exp over column tiles, token loss, per-block module sums ----------
@@ -214,19 +322,24 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
   const int k = blockIdx.y;
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int64_t n = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+  // compacted: the module's kept tokens are rows [offsets[k], offsets[k + 1])
+  const bool compact = a.kept_local != nullptr;
+  const int64_t row = compact ? a.offsets[k] + n : static_cast<int64_t>(k) * a.N + n;
+  const bool in_module = compact ? row < a.offsets[k + 1] : n < a.N;
   double lsum = 0.0, tsum = 0.0;
   int cnt = 0;
   int bad = 0;
-  if (n < a.N) {
-    const int64_t row = static_cast<int64_t>(k) * a.N + n;
+  if (in_module) {
+    const int64_t tok = compact ? a.orig_row[row] : row;     // the token's row of loss_tok
+    const int* tgt = compact ? a.tgt_c : a.targets;
     float mx = -INFINITY, s = 0.f, us = 0.f;
     int best_tile = 0;
     // E_p[s] - s_y = e^{M - lse} sum_t e^{m_t - M} (u_t - s_y s_t), with the
     // target's term left out of the tile sums s_t and u_t = sum of exp(z - m_t) s
     float ys = 0.f;
     if constexpr (!kExit) {
-      const int y0 = a.targets ? a.targets[row] : a.ignore_index;
-      if (token_kept(a, row, y0)) ys = kHeads ? a.sy[row] : a.zy[row];
+      const int y0 = tgt ? tgt[row] : a.ignore_index;
+      if (compact || token_kept(a, row, y0)) ys = kHeads ? a.sy[row] : a.zy[row];
     }
     for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
       float2 st[8];
@@ -256,9 +369,9 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       }
       mx = cm;
     }
-    const int y = a.targets ? a.targets[row] : a.ignore_index;
-    bad = !(y >= 0 && y < a.V) && y != a.ignore_index;
-    const bool kept = token_kept(a, row, y);
+    const int y = tgt ? tgt[row] : a.ignore_index;
+    bad = !compact && !(y >= 0 && y < a.V) && y != a.ignore_index;
+    const bool kept = compact || token_kept(a, row, y);
     float l = mx + logf(s), nll = 0.f;
     if constexpr (kExit) {
       if (a.top1 && in_bounds(best_tile < a.n_tiles_v, a.flags))
@@ -277,7 +390,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       a.lse[row] = l;
     }
     const float loss = kept ? nll : 0.f;
-    if (a.loss_tok) a.loss_tok[row] = loss;
+    if (a.loss_tok) a.loss_tok[tok] = loss;
     lsum = loss;
     cnt = kept ? 1 : 0;
     if constexpr (!kExit) {
@@ -364,11 +477,17 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int64_t row = blockIdx.x;
   if (!in_bounds(row < M, a.flags)) return;
-  const int k = static_cast<int>(row / a.N);
-  const int y = a.targets[row];
   uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
   const int nvec = a.ldp / 8;
-  if (!token_kept(a, row, y)) {
+  // compacted: rows [0, Mk) are kept tokens; past them, the rows up to
+  // offsets[K-1] + N are zeroed (the dW product reduces over them), the rest is
+  // never read
+  const bool compact = a.kept_local != nullptr;
+  if (compact && row >= a.offsets[a.K - 1] + a.N) return;
+  const int64_t tok = compact ? a.orig_row[row < a.offsets[a.K] ? row : 0] : row;
+  const int k = static_cast<int>(tok / a.N);
+  const int y = compact ? a.tgt_c[row < a.offsets[a.K] ? row : 0] : a.targets[row];
+  if (compact ? row >= a.offsets[a.K] : !token_kept(a, row, y)) {
     for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
     return;
   }
@@ -409,9 +528,17 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int k = blockIdx.y / a.db_chunks;
   const int chunk = blockIdx.y - k * a.db_chunks;
-  const int64_t row0 = static_cast<int64_t>(k) * a.N + static_cast<int64_t>(chunk) * kGradRows;
-  const int64_t left = static_cast<int64_t>(k + 1) * a.N - row0;
-  const int rows = left < kGradRows ? static_cast<int>(left) : kGradRows;
+  // compacted: module k's kept tokens are rows [offsets[k], offsets[k + 1]); the
+  // final module's chunks also zero the rows past Mk up to offsets[K-1] + N,
+  // which the dW product reads
+  const bool compact = a.kept_local != nullptr;
+  const int64_t mbase = compact ? a.offsets[k] : static_cast<int64_t>(k) * a.N;
+  const int64_t mkept = compact ? a.offsets[k + 1] : mbase + a.N;
+  const int64_t row0 = mbase + static_cast<int64_t>(chunk) * kGradRows;
+  const int64_t left = mbase + a.N - row0;
+  const int64_t end = (compact && k < a.K - 1) ? mkept : mbase + a.N;
+  const int rows = row0 >= end ? 0 : static_cast<int>(end - row0 < kGradRows ? end - row0 : kGradRows);
+  (void)left;
   const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
   if (!in_bounds(k < a.K && row0 + rows <= M, a.flags)) return;
   const float w = a.inv_nvalid[k];
@@ -419,8 +546,8 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   if (threadIdx.x < rows) {
     const int r = threadIdx.x;
     const int64_t i = row0 + r;
-    const int y = a.targets[i];
-    const bool kept = token_kept(a, i, y);
+    const int y = compact ? (i < mkept ? a.tgt_c[i] : -1) : a.targets[i];
+    const bool kept = compact ? i < mkept : token_kept(a, i, y);
     const float l = a.lse[i];
     const float wr = kept ? w : 0.f;
 #pragma unroll
@@ -495,8 +622,16 @@ __global__ void __launch_bounds__(256) dgamma_reduce_kernel(const RowArgs a) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int j = blockIdx.x * 32 + lane;
-  const int seg = (a.dg_chunks + 7) / 8;
-  const int c1 = min(a.dg_chunks, (warp + 1) * seg);
+  // compacted: the final module's kept tokens are rows [offsets[K-1], Mk), so
+  // the 32-row blocks holding them are fewer than for all its tokens
+  int chunks = a.dg_chunks;
+  if (a.kept_local != nullptr) {
+    const int64_t f0 = a.offsets[a.K - 1], f1 = a.offsets[a.K];
+    chunks = f1 > f0 ? static_cast<int>(((f1 - 1) >> 5) - (f0 >> 5) + 1) : 0;
+    chunks = min(chunks, a.dg_chunks);
+  }
+  const int seg = (chunks + 7) / 8;
+  const int c1 = min(chunks, (warp + 1) * seg);
   float acc = 0.f;
   if (j < a.d) {
     int c = warp * seg;
@@ -540,6 +675,14 @@ cudaError_t launch_rmsnorm_fwd(const RowArgs& a, cudaStream_t s) {
     case 8: rmsnorm_fwd_kernel<8><<<grid, 256, 0, s>>>(a); break;
     default: rmsnorm_fwd_kernel<0><<<grid, 256, 0, s>>>(a); break;
   }
+  return launched();
+}
+
+cudaError_t launch_keep_scan(const RowArgs& a, cudaStream_t s) {
+  keep_scan_kernel<<<dim3(a.nchunks, a.K), kScanRows, 0, s>>>(a);
+  cudaError_t e = launched();
+  if (e != cudaSuccess) return e;
+  keep_offsets_kernel<<<1, 1024, 0, s>>>(a);
   return launched();
 }
 

@@ -61,7 +61,9 @@ struct Layout {
   size_t inv_nvalid = 0;
   size_t stats = 0, xhat = 0, P = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
+  size_t kept_local = 0, chunk_base = 0, offsets = 0, orig_row = 0, tgt_c = 0;
   int aux_slots = 0;
+  int nchunks = 0;
 };
 
 solo_status_t check_dims(const solo_dims_t* d) {
@@ -87,9 +89,9 @@ Layout make_layout(const solo_dims_t& d) {
   L.ldp = static_cast<int>(align_up(d.V, 8));
   L.n_tiles_v = (d.V + kBN - 1) / kBN;
   L.part_blocks = static_cast<int>((d.N + 255) / 256);
-  // dgamma partial sums per 32-row block holding rows of the final module
-  const int64_t row0_final = static_cast<int64_t>(d.K - 1) * d.N;
-  L.dg_chunks = static_cast<int>(((L.M - 1) >> 5) - (row0_final >> 5) + 1);
+  // dgamma partial sums per 32-row block holding rows of the final module: its
+  // kept tokens start at any compact row, so they span at most N/32 + 1 blocks
+  L.dg_chunks = static_cast<int>((d.N + 31) / 32 + 1);
   L.db_chunks = static_cast<int>((d.N + kGradRows - 1) / kGradRows);
   const size_t M = static_cast<size_t>(L.M);
   size_t off = 0;
@@ -124,6 +126,14 @@ Layout make_layout(const solo_dims_t& d) {
   L.aux_slots = std::max(split_aux_slots(tiles_dx, (d.V + kBK - 1) / kBK, true),
                          split_aux_slots(tiles_dw, (d.N + kBK - 1) / kBK, false));
   L.aux = take(static_cast<size_t>(std::max(L.aux_slots, 1)) * 2 * kBM * kBN * 4);
+  // kept-token compaction: in-chunk ranks, chunk prefixes, module offsets, the
+  // token and target of every compact row
+  L.nchunks = static_cast<int>((d.N + kScanRows - 1) / kScanRows);
+  L.kept_local = take(M * 4);
+  L.chunk_base = take(static_cast<size_t>(d.K) * L.nchunks * 4);
+  L.offsets = take((SOLO_MAX_MODULES + 1) * 4);
+  L.orig_row = take(M * 4);
+  L.tgt_c = take(M * 4);
   L.total = off;
   return L;
 }
@@ -328,6 +338,13 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.dbias = dbias;
   ra.db_part = reinterpret_cast<float*>(ws + L.db_part);
   ra.db_chunks = L.db_chunks;
+  // masked tokens are skipped: the kept ones are compacted into rows [0, Mk)
+  ra.kept_local = reinterpret_cast<int32_t*>(ws + L.kept_local);
+  ra.chunk_base = reinterpret_cast<int32_t*>(ws + L.chunk_base);
+  ra.nchunks = L.nchunks;
+  ra.offsets = reinterpret_cast<int32_t*>(ws + L.offsets);
+  ra.orig_row = reinterpret_cast<int32_t*>(ws + L.orig_row);
+  ra.tgt_c = reinterpret_cast<int32_t*>(ws + L.tgt_c);
 
   const uint64_t M = static_cast<uint64_t>(L.M);
   const uint64_t d = static_cast<uint64_t>(D.d);
@@ -359,7 +376,9 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
 
   if (clear_flags && fail(cudaMemsetAsync(ra.flags, 0, 256, stream))) return SOLO_ERR_CUDA;
 
-  if (!mark(SOLO_STAGE_RMSNORM) || fail(launch_rmsnorm_fwd(ra, stream))) return SOLO_ERR_CUDA;
+  if (!mark(SOLO_STAGE_RMSNORM) || fail(launch_keep_scan(ra, stream)) ||
+      fail(launch_rmsnorm_fwd(ra, stream)))
+    return SOLO_ERR_CUDA;
 
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
@@ -371,7 +390,9 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   g.n_blocks = L.n_tiles_v;
   g.group_m = kGroupLogits;
   g.num_tiles = g.m_blocks * g.n_blocks;
-  g.targets = targets;
+  g.targets = ra.tgt_c;             // compact rows: kept tokens only
+  g.m_dev = ra.offsets + D.K;       // their count
+  g.orig_row = ra.orig_row;
   g.stats = ra.stats;
   g.zy = ra.zy;
   g.V = D.V;
@@ -412,6 +433,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.dg_part = dgamma ? ra.dgamma_part : nullptr;
   gx.dg_blocks = L.dg_chunks;
   gx.dg_row0 = static_cast<int64_t>(D.K - 1) * D.N;
+  gx.row0_dev = ra.offsets + (D.K - 1);   // the final module's first kept token
   gx.aux_part0 = 1;     // cut tiles: every part to a slot, summed by cut_tiles_norm
   plan_units(gx, sms, true);
   // whole tiles write dH from TMEM and cut tiles write slots: the output map
@@ -434,6 +456,11 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
     gw.group_m = kGroupDW;
     gw.num_tiles = gw.m_blocks * gw.n_blocks;
     gw.aux_part0 = 0;
+    // the reduction runs over rows [offsets[K-1], offsets[K-1] + N): the final
+    // module's kept tokens, then zeroed rows (masked tokens' share of [Mk, M))
+    gw.m_dev = nullptr;
+    gw.row0_dev = ra.offsets + (D.K - 1);
+    gw.orig_row = nullptr;
     plan_units(gw, sms, true);
     if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, mAux, gw, sms, stream)) ||
         fail(launch_split_fixup(gw, dW, D.d, aux, stream)))

@@ -74,6 +74,37 @@ MULTIWAVE = [
 ]
 
 
+# Masked tokens are skipped by every product (the kept ones are compacted into
+# the first rows): most tokens masked, a final module with a few kept tokens
+# whose compact rows start off a 32-row boundary, every token of a module kept.
+MASKED = [
+    Workload("k3_n700_d264_v1500_mask90", K=3, N=700, d=264, V=1500, seed=53, mask_frac=0.9,
+             row_scale=True),
+    Workload("k4_n2000_d512_v3000_mask37", K=4, N=2000, d=512, V=3000, seed=54,
+             mask_frac=0.37, targets="zipf"),
+]
+
+
+@pytest.mark.parametrize("wl", MASKED, ids=lambda w: w.name)
+def test_masked_tokens_skipped_full_parity(wl):
+    _, gpu, ref = _case(wl)
+    assert gpu["flags"] == 0
+    parity.compare_full(wl, gpu, ref)
+
+
+def test_all_tokens_masked():
+    """Nothing kept anywhere: every loss and gradient is exactly zero."""
+    wl = Workload("k2_n300_d128_v900_none", K=2, N=300, d=128, V=900, seed=55)
+    inp = synth.generate(wl)
+    tg = np.full_like(inp.targets, wl.ignore_index)
+    gpu = parity.run_gpu(wl, inp, targets=tg)
+    assert gpu["flags"] == 0
+    assert not np.any(gpu["loss_tok"]) and not np.any(gpu["loss_mean"])
+    for k in range(wl.K):
+        assert not np.any(gpu["dhidden"][k])
+    assert not np.any(gpu["dW"]) and not np.any(gpu["dgamma"])
+
+
 @pytest.mark.parametrize("wl", MULTIWAVE, ids=lambda w: w.name)
 def test_multiwave_full_parity(wl):
     """Element-by-element parity where every persistent GEMM loops over many
@@ -182,12 +213,12 @@ def test_kernel_launch_counter():
 
     full = count()
     assert full == count()
-    # rmsnorm, logits, lse, module means, grad, dxhat (with the RMSNorm backward),
-    # dW, dgamma reduce: 8, plus per product whose last wave was cut a fix-up,
-    # and for dX̂ the RMSNorm backward of its cut tiles
-    assert 8 <= full <= 11
+    # kept-token scan and offsets, rmsnorm, logits, lse, module means, grad, dxhat
+    # (with the RMSNorm backward), dW, dgamma reduce: 10, plus the dW fix-up when
+    # its last wave was cut and the RMSNorm backward of dX̂'s cut tiles
+    assert 10 <= full <= 12
     # without dW and dgamma: no dW GEMM (nor its fix-up) and no dgamma reduction
-    assert 6 <= count(want_dW=False, want_dgamma=False) <= full - 2
+    assert 8 <= count(want_dW=False, want_dgamma=False) <= full - 2
 
 
 def test_zero_readout_closed_forms():
