@@ -74,6 +74,9 @@ constexpr int kSmemTotal = kSmemMisc + 16 + 1024;   // + alignment slack
 static_assert(kSmemTotal <= 232448, "shared memory budget");
 
 constexpr float kLog2e = 1.4426950408889634f;
+// Exponentials are stored against the reference 0 while the tile's maximum logit
+// stays within this bound (e^64 leaves fp32 and bf16 room for 2^23 terms).
+constexpr float kRefBound = 64.f;
 
 constexpr uint16_t kBothCtas = 0x3;
 
@@ -171,12 +174,16 @@ struct NormRow {
   float r, coef;       // r_i and (r_i^3 / d) S_i
   const uint16_t* h;   // the row of hidden (bf16)
   uint16_t* dh;        // the row of dhidden (bf16)
+  // dxhat = fa acc - fb W_y: the accumulator holds the stored exponentials times
+  // W (a row left out of the gradient pass) or G W (fa = 1, fb = 0)
+  float fa, fb;
+  const uint16_t* wy;  // the row W_y, or null (fb = 0)
 };
 
 // dg_row0: first row of the final module (compacted rows: its first kept token).
 __device__ __forceinline__ NormRow norm_row(const GemmArgs& g, int64_t row, int M,
                                             int64_t dg_row0) {
-  NormRow nr{false, false, 0.f, 0.f, nullptr, nullptr};
+  NormRow nr{false, false, 0.f, 0.f, nullptr, nullptr, 1.f, 0.f, nullptr};
   if (row >= M) return nr;
   const int64_t tok = g.orig_row ? g.orig_row[row] : row;
   const int k = static_cast<int>(tok / g.tokens_per_module);
@@ -190,6 +197,19 @@ __device__ __forceinline__ NormRow norm_row(const GemmArgs& g, int64_t row, int 
   nr.coef = r * r * (tau * g.inv_nvalid[k] * g.edz[row]) / static_cast<float>(g.N);
   nr.h = g.hidden[k] + n * g.N;
   nr.dh = g.dhidden[k] + n * g.N;
+  if (g.row_fa != nullptr) {
+    const float fa = g.row_fa[row];
+    if (fa >= 0.f) {              // a row whose gradient is formed here
+      const float scale = tau * g.inv_nvalid[k];
+      nr.fa = scale * fa;
+      nr.fb = scale * g.row_fb[row];
+      const int y = g.targets[row];
+      if (nr.fb != 0.f && in_bounds(y >= 0 && y < g.Vw, g.flags))
+        nr.wy = g.W + static_cast<int64_t>(y) * g.N;
+      else
+        nr.fb = 0.f;
+    }
+  }
   return nr;
 }
 
@@ -217,10 +237,25 @@ __device__ __forceinline__ float reduce_scatter32(float (&p)[32]) {
 // of 8), dxhat in v: dH in bf16, and, when the warp holds rows of the final
 // module (dg_warp, warp-uniform), the column sums over its 32 rows of
 // dxhat h r, lane j storing column col0 + j at dg_dst[j].
-__device__ __forceinline__ void norm_bwd_chunk(const GemmArgs& g, const float (&v)[32], int col0,
+__device__ __forceinline__ void norm_bwd_chunk(const GemmArgs& g, float (&v)[32], int col0,
                                                int cols, const NormRow& nr, bool dg_warp,
                                                float* dg_dst) {
   const int lane = threadIdx.x & 31;
+  if (nr.fa != 1.f || nr.wy != nullptr) {
+    // dxhat = fa acc - fb W_y
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 wv = make_uint4(0, 0, 0, 0);
+      if (nr.wy != nullptr && 8 * q < cols) wv = __ldg(reinterpret_cast<const uint4*>(nr.wy + col0) + q);
+      const uint32_t ww[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int c = 8 * q + 2 * j;
+        v[c] = fmaf(nr.fa, v[c], -nr.fb * __uint_as_float(ww[j] << 16));
+        v[c + 1] = fmaf(nr.fa, v[c + 1], -nr.fb * __uint_as_float(ww[j] & 0xFFFF0000u));
+      }
+    }
+  }
   float h[32], gm[32];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -627,8 +662,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           mx = fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]),
                      fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
         }
-        const float mlog = mx * kLog2e;
-        // the sums of exp(z - m) and of exp(z - m) s, each in the two lanes of a
+        // The tile's exponentials are taken against a reference shared by all the
+        // row's tiles, 0, unless the tile's maximum lies beyond +-kRefBound (then
+        // the maximum itself): a row all of whose tiles use 0 has a gradient that
+        // is its stored exponentials times one factor per row, which the dX̂
+        // epilogue applies; only the other rows need the gradient pass.
+        const float ref = fabsf(mx) > kRefBound ? mx : 0.f;
+        const float mlog = ref * kLog2e;
+        // the sums of exp(z - ref) and of exp(z - ref) s, each in the two lanes of a
         // packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
         float2 uacc = make_float2(0.f, 0.f);
@@ -707,7 +748,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         }
         const float ssum = sacc.x + sacc.y;
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
-          args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
+          args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(ref, ssum);
           args.usum[static_cast<size_t>(nb) * args.M + row] = uacc.x + uacc.y;
         }
         if constexpr (kHeads) {

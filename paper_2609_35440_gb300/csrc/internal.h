@@ -128,6 +128,13 @@ struct GemmArgs {
   const int32_t* orig_row;  // [M]: token (k * N + n) of a row, or null (the row itself)
   int32_t sms;              // multiprocessors, for the device-side plan
   int32_t split_ok;         // the plan may cut the last partial wave
+  // kDxhat: rows whose gradient the epilogue forms from the stored exponentials
+  // (exp(z) against the reference 0): dxhat = tau/Nvalid (fa acc - fb W_y).
+  // fa < 0 marks a row the gradient pass has turned into G (fa = 1, fb = 0).
+  const float* row_fa;      // [M] e^{-lse}, or -1; null: every row is G
+  const float* row_fb;      // [M] 1 - p_y
+  const uint16_t* W;        // [V, d] for W_y
+  int32_t Vw;               // V
 };
 
 size_t gemm_smem_bytes();
@@ -258,6 +265,14 @@ struct RowArgs {
   float* dbias;          // [K, V] or null
   float* db_part;        // [K, db_chunks, ldp]
   int32_t db_chunks;     // row chunks per module of the gradient pass
+  // Rows whose gradient the dX̂ epilogue forms (the log-sum-exp pass decides):
+  // row_fa = e^{-lse} and row_fb = 1 - p_y for them, row_fa = -1 for the rows
+  // the gradient pass turns into G (the final module's, whose dW needs G, and
+  // rows with a tile stored against its own maximum or lse above 60).  Null:
+  // every row goes through the gradient pass.
+  float* row_fa;         // [M]
+  float* row_fb;         // [M]
+  int32_t full_grad;     // 1: every row through the gradient pass (bias gradients)
   // Compaction of the kept tokens (null kept_local: every token keeps its row).
   // Kept tokens take rows [0, Mk) of the per-row buffers in token order, module
   // by module; each masked token zeroes one row of [Mk, M).

@@ -334,6 +334,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     const int* tgt = compact ? a.tgt_c : a.targets;
     float mx = -INFINITY, s = 0.f, us = 0.f;
     int best_tile = 0;
+    bool own_ref = false;       // a tile stored against its own maximum, not 0
     // E_p[s] - s_y = e^{M - lse} sum_t e^{m_t - M} (u_t - s_y s_t), with the
     // target's term left out of the tile sums s_t and u_t = sum of exp(z - m_t) s
     float ys = 0.f;
@@ -355,6 +356,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       for (int u = 0; u < 8; ++u) {
         if (kExit && st[u].x > cm) best_tile = t0 + u;   // strict: the first tile with the max
         cm = fmaxf(cm, st[u].x);
+        if (!kExit && t0 + u < a.n_tiles_v && st[u].x != 0.f) own_ref = true;
       }
       const float rescale = expf(mx - cm);  // mx = -inf only before the first tile (s = 0)
       s *= rescale;
@@ -400,6 +402,17 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       const float e = kept ? us * expf(mx - l) : 0.f;   // the sums are relative to mx
       a.edz[row] = e;
       if constexpr (kHeads) tsum = e;
+      if (a.row_fa != nullptr) {
+        // An auxiliary row whose tiles all used the reference 0: its gradient is
+        // tau/Nvalid (e^{-lse} P - (1 - p_y) e_y) with P the stored exponentials,
+        // formed by the dX̂ epilogue (e^{-lse} kept well inside fp32 by lse <= 60).
+        // The final module's rows (dW needs G) and the rest go through the
+        // gradient pass.
+        const int kk = static_cast<int>(tok / a.N);
+        const bool factor = kept && !a.full_grad && kk < a.K - 1 && !own_ref && l <= 60.f;
+        a.row_fa[row] = factor ? expf(-l) : -1.f;
+        a.row_fb[row] = factor ? -expm1f(-nll) : 0.f;
+      }
     }
   }
   if (__syncthreads_or(bad) && threadIdx.x == 0) atomicOr(a.flags, SOLO_FLAG_BAD_TARGET);
@@ -484,6 +497,8 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   // never read
   const bool compact = a.kept_local != nullptr;
   if (compact && row >= a.offsets[a.K - 1] + a.N) return;
+  // rows whose gradient the dX̂ epilogue forms keep their stored exponentials
+  if (a.row_fa != nullptr && (!compact || row < a.offsets[a.K]) && a.row_fa[row] >= 0.f) return;
   const int64_t tok = compact ? a.orig_row[row < a.offsets[a.K] ? row : 0] : row;
   const int k = static_cast<int>(tok / a.N);
   const int y = compact ? a.tgt_c[row < a.offsets[a.K] ? row : 0] : a.targets[row];

@@ -62,6 +62,7 @@ struct Layout {
   size_t stats = 0, xhat = 0, P = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
   size_t kept_local = 0, chunk_base = 0, offsets = 0, orig_row = 0, tgt_c = 0;
+  size_t row_fa = 0, row_fb = 0;
   int aux_slots = 0;
   int nchunks = 0;
 };
@@ -134,6 +135,9 @@ Layout make_layout(const solo_dims_t& d) {
   L.offsets = take((SOLO_MAX_MODULES + 1) * 4);
   L.orig_row = take(M * 4);
   L.tgt_c = take(M * 4);
+  // per-row factors of the rows whose gradient the dX̂ epilogue forms
+  L.row_fa = take(M * 4);
+  L.row_fb = take(M * 4);
   L.total = off;
   return L;
 }
@@ -345,6 +349,11 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.offsets = reinterpret_cast<int32_t*>(ws + L.offsets);
   ra.orig_row = reinterpret_cast<int32_t*>(ws + L.orig_row);
   ra.tgt_c = reinterpret_cast<int32_t*>(ws + L.tgt_c);
+  // the auxiliary modules' gradients are formed in the dX̂ epilogue where the
+  // stored exponentials allow it; with bias gradients every row takes the pass
+  ra.row_fa = reinterpret_cast<float*>(ws + L.row_fa);
+  ra.row_fb = reinterpret_cast<float*>(ws + L.row_fb);
+  ra.full_grad = dbias != nullptr ? 1 : 0;
 
   const uint64_t M = static_cast<uint64_t>(L.M);
   const uint64_t d = static_cast<uint64_t>(D.d);
@@ -434,6 +443,10 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   gx.dg_blocks = L.dg_chunks;
   gx.dg_row0 = static_cast<int64_t>(D.K - 1) * D.N;
   gx.row0_dev = ra.offsets + (D.K - 1);   // the final module's first kept token
+  gx.row_fa = ra.row_fa;
+  gx.row_fb = ra.row_fb;
+  gx.W = W;
+  gx.Vw = D.V;
   gx.aux_part0 = 1;     // cut tiles: every part to a slot, summed by cut_tiles_norm
   plan_units(gx, sms, true);
   // whole tiles write dH from TMEM and cut tiles write slots: the output map
