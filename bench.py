@@ -547,16 +547,18 @@ def run_ours(args, wl):
         "config": {"workload": wl.name, "K": wl.K, "N": wl.N, "d": wl.d, "V": wl.V,
                    "global_batch_tokens": world * wl.M, "parallelism": f"replicas{world}",
                    "l2": l2_note(wl, True)},
+        # the paper's count, (2K+1) 2NVd over every token of the call, per second
+        # (a rate, not a fraction of peak: masked tokens are skipped)
         "algo_tflops": algo / step_s / 1e12,
-        # the whole call's algorithmic rate against the same peak as the roofline
-        "algo_frac_of_peak": algo / step_s / 1e12 / peak,
-        # the paper's work on kept tokens only (masked tokens still run through
-        # every product; the mean loss counts kept tokens)
+        # the paper's work on the kept tokens (the mean loss counts kept tokens),
+        # against the same peak as the roofline: the whole call's fraction
         "kept_algo_tflops": kept / step_s / 1e12,
         "kept_algo_frac_of_peak": kept / step_s / 1e12 / peak,
         # what the tensor cores execute: no logits are recomputed (the forward
-        # stores its exponentials) and masked tokens are skipped
+        # stores its exponentials), masked tokens are skipped except in dW's
+        # reduction over the final module's N rows
         "executed_tflops": executed / step_s / 1e12,
+        "executed_frac_of_peak": executed / step_s / 1e12 / peak,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
         "roofline": {"bound": "tensor",
                      "kernel": ("auxiliary on-chip pass (tcgen05, cluster split of d)"
