@@ -403,15 +403,18 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       a.edz[row] = e;
       if constexpr (kHeads) tsum = e;
       if (a.row_fa != nullptr) {
-        // An auxiliary row whose tiles all used the reference 0: its gradient is
-        // tau/Nvalid (e^{-lse} P - (1 - p_y) e_y) with P the stored exponentials,
-        // formed by the dX̂ epilogue (e^{-lse} kept well inside fp32 by lse <= 60).
-        // The final module's rows (dW needs G) and the rest go through the
-        // gradient pass.
+        // A row whose tiles all used the reference 0: its gradient is
+        // tau/Nvalid (e^{-lse} P - (1 - p_y) e_y) with P the stored exponentials
+        // (e^{-lse} kept well inside fp32 by lse <= 60).  An auxiliary row's is
+        // formed by the dX̂ epilogue (fb = 1 - p_y: the W_y term).  A final-module
+        // row's target entry of P becomes -(1 - p_y) e^{lse} in the gradient
+        // pass, so that tau/Nvalid e^{-lse} P is its whole G row (fb = 0).  The
+        // other rows (and every row when bias gradients are wanted) have the
+        // gradient pass turn P into G.
         const int kk = static_cast<int>(tok / a.N);
-        const bool factor = kept && !a.full_grad && kk < a.K - 1 && !own_ref && l <= 60.f;
+        const bool factor = kept && !a.full_grad && !own_ref && l <= 60.f;
         a.row_fa[row] = factor ? expf(-l) : -1.f;
-        a.row_fb[row] = factor ? -expm1f(-nll) : 0.f;
+        a.row_fb[row] = (factor && kk < a.K - 1) ? -expm1f(-nll) : 0.f;
       }
     }
   }
@@ -497,8 +500,30 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   // never read
   const bool compact = a.kept_local != nullptr;
   if (compact && row >= a.offsets[a.K - 1] + a.N) return;
-  // rows whose gradient the dX̂ epilogue forms keep their stored exponentials
-  if (a.row_fa != nullptr && (!compact || row < a.offsets[a.K]) && a.row_fa[row] >= 0.f) return;
+  if (a.row_fa != nullptr && (!compact || row < a.offsets[a.K]) && a.row_fa[row] >= 0.f) {
+    // rows whose gradient is P times a per-row factor keep their exponentials;
+    // a final-module row (dW = G^T xhat) gets its target entry and its xhat row
+    // scaled by that factor, tau/Nvalid e^{-lse}: G^T xhat = P'^T (c xhat)
+    const int64_t rk = compact ? row : row;
+    const bool final_row = compact ? rk >= a.offsets[a.K - 1] : rk >= static_cast<int64_t>(a.K - 1) * a.N;
+    if (!final_row) return;
+    const int64_t tk = compact ? a.orig_row[rk] : rk;
+    const int kf = static_cast<int>(tk / a.N);
+    const int yf = compact ? a.tgt_c[rk] : a.targets[rk];
+    const float tauf = a.tau ? a.tau[kf] : 1.f;
+    const float c = tauf * a.inv_nvalid[kf] * a.row_fa[rk];
+    if (threadIdx.x == 0 && in_bounds(yf >= 0 && yf < a.V, a.flags))
+      a.P[rk * a.ldp + yf] = __bfloat16_as_ushort(__float2bfloat16(expm1f(-a.nll[rk]) * expf(a.lse[rk])));
+    uint4* xr = reinterpret_cast<uint4*>(a.xhat + rk * a.d);
+    for (int v = threadIdx.x; v < a.d / 8; v += 256) {
+      float f[8];
+      unpack8(xr[v], f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) f[j] *= c;
+      xr[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+    }
+    return;
+  }
   const int64_t tok = compact ? a.orig_row[row < a.offsets[a.K] ? row : 0] : row;
   const int k = static_cast<int>(tok / a.N);
   const int y = compact ? a.tgt_c[row < a.offsets[a.K] ? row : 0] : a.targets[row];
