@@ -85,14 +85,22 @@ constexpr uint16_t kBothCtas = 0x3;
 // host's rule (plan_units): whole tiles fill complete waves of pairs, the rest
 // is cut along the reduction.
 struct Plan {
-  int M, m_blocks, num_tiles, full_tiles, split, num_units;
+  int M, m_blocks, num_tiles, full_tiles, split, num_units, k_blocks;
 };
 
 __device__ __forceinline__ Plan make_plan(const GemmArgs& a) {
-  Plan p{a.M, a.m_blocks, a.num_tiles, a.full_tiles, a.split, a.num_units};
-  if (a.m_dev == nullptr) return p;
-  p.M = min(*a.m_dev, a.M);
-  p.m_blocks = (p.M + 2 * kBM - 1) / (2 * kBM);
+  Plan p{a.M, a.m_blocks, a.num_tiles, a.full_tiles, a.split, a.num_units, a.k_blocks};
+  if (a.m_dev == nullptr && a.kend_dev == nullptr) return p;
+  if (a.m_dev != nullptr) {
+    p.M = min(*a.m_dev, a.M);
+    p.m_blocks = (p.M + 2 * kBM - 1) / (2 * kBM);
+  }
+  if (a.kend_dev != nullptr && a.row0_dev != nullptr) {
+    // kDW over the final module's kept tokens (all masked: the host's length
+    // over zeroed rows)
+    const int rows = *a.kend_dev - *a.row0_dev;
+    if (rows > 0) p.k_blocks = min((rows + kBK - 1) / kBK, a.k_blocks);
+  }
   p.num_tiles = p.m_blocks * a.n_blocks;
   p.full_tiles = p.num_tiles;
   p.split = 1;
@@ -100,7 +108,7 @@ __device__ __forceinline__ Plan make_plan(const GemmArgs& a) {
   const int pairs = min(max(a.sms / 2, 1), kMaxAuxSlots + 1);
   const int rem = p.num_tiles % pairs;
   if (!a.split_ok || rem == 0) return p;
-  int s = min(min(pairs / rem, kMaxSplit), a.k_blocks);
+  int s = min(min(pairs / rem, kMaxSplit), p.k_blocks);
   while (s > 1 && rem * (a.aux_part0 ? s : s - 1) > min(a.aux_slots, kMaxAuxSlots)) --s;
   if (s < 2) return p;
   p.full_tiles = p.num_tiles - rem;
@@ -128,14 +136,14 @@ __device__ __forceinline__ void unit_range(int u, const GemmArgs& a, const Plan&
     t = u;
     part = 0;
     kb_lo = 0;
-    kb_hi = a.k_blocks;
+    kb_hi = p.k_blocks;
     return;
   }
   const int i = u - p.full_tiles;
   t = p.full_tiles + i / p.split;
   part = i % p.split;
-  kb_lo = static_cast<int>(static_cast<int64_t>(part) * a.k_blocks / p.split);
-  kb_hi = static_cast<int>(static_cast<int64_t>(part + 1) * a.k_blocks / p.split);
+  kb_lo = static_cast<int>(static_cast<int64_t>(part) * p.k_blocks / p.split);
+  kb_hi = static_cast<int>(static_cast<int64_t>(part + 1) * p.k_blocks / p.split);
 }
 
 // Waits without looking at the abort flag, bounded in time: used to drain

@@ -126,6 +126,9 @@ struct GemmArgs {
   const int32_t* row0_dev;  // kDW: first reduction row / kDxhat: first row of the final
                             //   module (dgamma blocks), or null (k_row0 / dg_row0)
   const int32_t* orig_row;  // [M]: token (k * N + n) of a row, or null (the row itself)
+  const int32_t* kend_dev;  // kDW: end of the reduction rows (the kept tokens' count):
+                            //   the device plan reduces over [*row0_dev, *kend_dev)
+                            //   rounded up to whole blocks, or null (k_blocks)
   int32_t sms;              // multiprocessors, for the device-side plan
   int32_t split_ok;         // the plan may cut the last partial wave
   // kDxhat: rows whose gradient the epilogue forms from the stored exponentials

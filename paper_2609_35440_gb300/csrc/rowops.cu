@@ -495,16 +495,17 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
   if (!in_bounds(row < M, a.flags)) return;
   uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
   const int nvec = a.ldp / 8;
-  // compacted: rows [0, Mk) are kept tokens; past them, the rows up to
-  // offsets[K-1] + N are zeroed (the dW product reduces over them), the rest is
+  // compacted: rows [0, Mk) are kept tokens; past them, the rows up to the
+  // final module's first row plus N rounded up to whole 128-row reduction
+  // blocks are zeroed (the dW product's reduction may read them), the rest is
   // never read
   const bool compact = a.kept_local != nullptr;
-  if (compact && row >= a.offsets[a.K - 1] + a.N) return;
+  if (compact && row >= a.offsets[a.K - 1] + (a.N + 127) / 128 * 128) return;
   if (a.row_fa != nullptr && (!compact || row < a.offsets[a.K]) && a.row_fa[row] >= 0.f) {
     // rows whose gradient is P times a per-row factor keep their exponentials;
     // a final-module row (dW = G^T xhat) gets its target entry and its xhat row
     // scaled by that factor, tau/Nvalid e^{-lse}: G^T xhat = P'^T (c xhat)
-    const int64_t rk = compact ? row : row;
+    const int64_t rk = row;
     const bool final_row = compact ? rk >= a.offsets[a.K - 1] : rk >= static_cast<int64_t>(a.K - 1) * a.N;
     if (!final_row) return;
     const int64_t tk = compact ? a.orig_row[rk] : rk;
@@ -569,16 +570,16 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   const int k = blockIdx.y / a.db_chunks;
   const int chunk = blockIdx.y - k * a.db_chunks;
   // compacted: module k's kept tokens are rows [offsets[k], offsets[k + 1]); the
-  // final module's chunks also zero the rows past Mk up to offsets[K-1] + N,
-  // which the dW product reads
+  // final module's chunks also zero the rows past Mk up to its first row plus N
+  // rounded up to whole 128-row reduction blocks, which the dW product may read
+  // (their contents are stale: written as zeros, never scaled)
   const bool compact = a.kept_local != nullptr;
   const int64_t mbase = compact ? a.offsets[k] : static_cast<int64_t>(k) * a.N;
   const int64_t mkept = compact ? a.offsets[k + 1] : mbase + a.N;
   const int64_t row0 = mbase + static_cast<int64_t>(chunk) * kGradRows;
-  const int64_t left = mbase + a.N - row0;
-  const int64_t end = (compact && k < a.K - 1) ? mkept : mbase + a.N;
+  const int64_t end = (compact && k < a.K - 1) ? mkept
+                      : compact ? min(M, mbase + (a.N + 127) / 128 * 128) : mbase + a.N;
   const int rows = row0 >= end ? 0 : static_cast<int>(end - row0 < kGradRows ? end - row0 : kGradRows);
-  (void)left;
   const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
   if (!in_bounds(k < a.K && row0 + rows <= M, a.flags)) return;
   const float w = a.inv_nvalid[k];
@@ -620,12 +621,13 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
       const int r = r0 + u;
       if (r >= rows) break;
       const float c = cfac[r][tt];
+      const bool live = sy[r] >= 0;
       const int ycol = sy[r] - col0;
       float f[8];
       unpack8(in[u], f);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        float g = f[j] * c;
+        float g = live ? f[j] * c : 0.f;
         if (j == ycol) g = sgy[r];
         if (col0 + j >= a.V) g = 0.f;
         colsum[j] += g;

@@ -473,6 +473,7 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
     // module's kept tokens, then zeroed rows (masked tokens' share of [Mk, M))
     gw.m_dev = nullptr;
     gw.row0_dev = ra.offsets + (D.K - 1);
+    gw.kend_dev = ra.offsets + D.K;       // the final module's kept tokens only
     gw.orig_row = nullptr;
     plan_units(gw, sms, true);
     if (fail(launch_gemm(kDW, mG_mn, mX_mn, mDW, mAux, gw, sms, stream)) ||
