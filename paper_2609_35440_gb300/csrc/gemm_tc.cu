@@ -630,123 +630,131 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               b[j] = (brow != nullptr && c * 32 + j < ncols) ? __ldg(brow + c * 32 + j) : 0.f;
           }
         };
-        float mx = -INFINITY, zyv = 0.f, syv = 0.f;
-        for (int c = 0; c < kBN / 32; ++c) {
-          if (c * 32 >= ncols) break;
-          float v[32], bb[32], z[32];
-          tmem_ld32(tbase + c * 32, v);
-          if constexpr (kHeads) load_bias(c, bb);
-#pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            if constexpr (kHeads) {
-              const float2 zz = __ffma2_rn(make_float2(tau, tau), make_float2(v[j], v[j + 1]),
-                                           make_float2(bb[j], bb[j + 1]));
-              z[j] = zz.x;
-              z[j + 1] = zz.y;
-            } else {
-              z[j] = v[j];
-              z[j + 1] = v[j + 1];
-            }
-          }
-          // the target logit, in the chunks holding some lane's target only
-          const int yc = has_y ? yrel - c * 32 : -1;
-          if (__any_sync(0xffffffffu, static_cast<unsigned>(yc) < 32u)) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              zyv = (j == yc) ? z[j] : zyv;
-              if constexpr (kHeads) syv = (j == yc) ? v[j] : syv;
-            }
-          }
-          if (c * 32 + 32 > ncols) {              // ragged last chunk (warp-uniform)
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (c * 32 + j >= ncols) z[j] = -INFINITY;
-          }
-          // max of mx and the 32 values: a tree of three-input maxima
-          float t[11];
-#pragma unroll
-          for (int i = 0; i < 10; ++i) t[i] = fmax3(z[3 * i], z[3 * i + 1], z[3 * i + 2]);
-          t[10] = fmax3(z[30], z[31], mx);
-          mx = fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]),
-                     fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
-        }
-        // The tile's exponentials are taken against a reference shared by all the
-        // row's tiles, 0, unless the tile's maximum lies beyond +-kRefBound (then
-        // the maximum itself): a row all of whose tiles use 0 has a gradient that
-        // is its stored exponentials times one factor per row, which the dX̂
-        // epilogue applies; only the other rows need the gradient pass.
-        const float ref = fabsf(mx) > kRefBound ? mx : 0.f;
-        const float mlog = ref * kLog2e;
+        // One pass over the accumulator takes the tile's exponentials against the
+        // reference 0 and finds its maximum on the way.  They are taken against a
+        // reference shared by all the row's tiles, 0, unless the tile's maximum
+        // lies beyond +-kRefBound (then the maximum itself): a row all of whose
+        // tiles use 0 has a gradient that is its stored exponentials times one
+        // factor per row, which the dX̂ epilogue applies; only the other rows need
+        // the gradient pass.  A warp holding such a row (rare) runs the pass again
+        // against the maximum once the first pass's stores have landed.
+        float mx = -INFINITY, zyv = 0.f, syv = 0.f, ref = 0.f;
         // the sums of exp(z - ref) and of exp(z - ref) s, each in the two lanes of a
         // packed pair (even and odd columns)
         float2 sacc = make_float2(0.f, 0.f);
         float2 uacc = make_float2(0.f, 0.f);
-        for (int cp = 0; cp < kBN / 64; ++cp) {
-          if (cp * 64 >= ncols) break;
-          if (lane == 0) bulk_wait_group_read<1>();
-          __syncwarp();
-          const uint32_t srow = smem_u32(ebuf + buf * kEpiBufBytes) + lane * 128;
+        for (int pass = 0; pass < 2; ++pass) {
+          const float mlog = ref * kLog2e;
+          mx = -INFINITY;
+          sacc = make_float2(0.f, 0.f);
+          uacc = make_float2(0.f, 0.f);
+          // the bias of the next chunk is loaded while this one is worked on
+          float bnext[32];
+          if constexpr (kHeads) load_bias(0, bnext);
+          for (int cp = 0; cp < kBN / 64; ++cp) {
+            if (cp * 64 >= ncols) break;
+            if (lane == 0) bulk_wait_group_read<1>();
+            __syncwarp();
+            const uint32_t srow = smem_u32(ebuf + buf * kEpiBufBytes) + lane * 128;
 #pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            const int c = 2 * cp + half;
-            float v[32], bb[32];
-            if (c * 32 < ncols) {
-              tmem_ld32(tbase + c * 32, v);
-              if constexpr (kHeads) load_bias(c, bb);
-            } else {
+            for (int half = 0; half < 2; ++half) {
+              const int c = 2 * cp + half;
+              float v[32], bb[32];
+              if (c * 32 < ncols) {
+                tmem_ld32(tbase + c * 32, v);
 #pragma unroll
-              for (int j = 0; j < 32; ++j) v[j] = bb[j] = 0.f;
-            }
-            uint32_t p[16];
-            const bool ragged = c * 32 + 32 > ncols;      // warp-uniform
-            float z[32];
+                for (int j = 0; j < 32; ++j) bb[j] = kHeads ? bnext[j] : 0.f;
+                if constexpr (kHeads) {
+                  if ((c + 1) * 32 < ncols) load_bias(c + 1, bnext);
+                }
+              } else {
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) {
-              float2 zz = make_float2(v[j], v[j + 1]);
-              if constexpr (kHeads)
-                zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[j], bb[j + 1]));
-              z[j] = zz.x;
-              z[j + 1] = zz.y;
-            }
-            // The target's own term is left out of the tile's sums and of the
-            // stored exponentials (the gradient pass writes the target entry
-            // itself): the log-sum-exp pass forms lse - z_y = log1p(sum over
-            // v != y of exp(z_v - z_y)), so that 1 - p_y and E_p[s] - s_y of a
-            // confident row do not cancel.
-            const int ycol = has_y ? yrel - c * 32 : -1;
-            if (__any_sync(0xffffffffu, static_cast<unsigned>(ycol) < 32u)) {
-#pragma unroll
-              for (int j = 0; j < 32; ++j) z[j] = j == ycol ? -INFINITY : z[j];
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const float2 a = __ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]),
-                                          make_float2(kLog2e, kLog2e), make_float2(-mlog, -mlog));
-              float e0 = ex2_approx(a.x);
-              float e1 = ex2_approx(a.y);
-              if (ragged) {
-                const int col = c * 32 + 2 * j;
-                e0 = col < ncols ? e0 : 0.f;
-                e1 = col + 1 < ncols ? e1 : 0.f;
+                for (int j = 0; j < 32; ++j) v[j] = bb[j] = 0.f;
               }
-              sacc = __fadd2_rn(sacc, make_float2(e0, e1));
-              uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
-              p[j] = pack_bf16x2(e0, e1);
-            }
+              uint32_t p[16];
+              const bool ragged = c * 32 + 32 > ncols;      // warp-uniform
+              float z[32];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const uint32_t chunk = static_cast<uint32_t>(half * 4 + u) ^ (lane & 7);
-              st_shared_v4(srow + (chunk << 4), p[4 * u], p[4 * u + 1], p[4 * u + 2],
-                           p[4 * u + 3]);
+              for (int j = 0; j < 32; j += 2) {
+                float2 zz = make_float2(v[j], v[j + 1]);
+                if constexpr (kHeads)
+                  zz = __ffma2_rn(make_float2(tau, tau), zz, make_float2(bb[j], bb[j + 1]));
+                z[j] = zz.x;
+                z[j + 1] = zz.y;
+              }
+              // the target logit, in the chunks holding some lane's target only
+              const int ycol = has_y ? yrel - c * 32 : -1;
+              const bool ychunk = __any_sync(0xffffffffu, static_cast<unsigned>(ycol) < 32u);
+              if (ychunk) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                  zyv = (j == ycol) ? z[j] : zyv;
+                  if constexpr (kHeads) syv = (j == ycol) ? v[j] : syv;
+                }
+              }
+              if (ragged) {                 // columns past N take no part in the max
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (c * 32 + j >= ncols) z[j] = -INFINITY;
+              }
+              // the running maximum (the target's logit included): a tree of
+              // three-input maxima
+              {
+                float t[11];
+#pragma unroll
+                for (int i = 0; i < 10; ++i) t[i] = fmax3(z[3 * i], z[3 * i + 1], z[3 * i + 2]);
+                t[10] = fmax3(z[30], z[31], mx);
+                mx = fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]),
+                           fmax3(t[6], t[7], fmax3(t[8], t[9], t[10])));
+              }
+              // The target's own term is left out of the tile's sums and of the
+              // stored exponentials (the gradient pass writes the target entry
+              // itself): the log-sum-exp pass forms lse - z_y = log1p(sum over
+              // v != y of exp(z_v - z_y)), so that 1 - p_y and E_p[s] - s_y of a
+              // confident row do not cancel.
+              if (ychunk) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) z[j] = j == ycol ? -INFINITY : z[j];
+              }
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float2 a = __ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]),
+                                            make_float2(kLog2e, kLog2e),
+                                            make_float2(-mlog, -mlog));
+                float e0 = ex2_approx(a.x);
+                float e1 = ex2_approx(a.y);
+                if (ragged) {
+                  const int col = c * 32 + 2 * j;
+                  e0 = col < ncols ? e0 : 0.f;
+                  e1 = col + 1 < ncols ? e1 : 0.f;
+                }
+                sacc = __fadd2_rn(sacc, make_float2(e0, e1));
+                uacc = __ffma2_rn(make_float2(e0, e1), make_float2(v[2 * j], v[2 * j + 1]), uacc);
+                p[j] = pack_bf16x2(e0, e1);
+              }
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const uint32_t chunk = static_cast<uint32_t>(half * 4 + u) ^ (lane & 7);
+                st_shared_v4(srow + (chunk << 4), p[4 * u], p[4 * u + 1], p[4 * u + 2],
+                             p[4 * u + 3]);
+              }
             }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + cp * 64, m0 + 32 * q);
+              bulk_commit_group();
+            }
+            buf ^= 1;
           }
-          fence_proxy_async_smem();
+          if (pass == 1) break;
+          const bool redo = fabsf(mx) > kRefBound;
+          if (!__any_sync(0xffffffffu, redo)) break;
+          ref = redo ? mx : 0.f;
+          // the second pass overwrites the stored tiles: the first pass's stores
+          // must have completed
+          if (lane == 0) bulk_wait_group<0>();
           __syncwarp();
-          if (lane == 0) {
-            tma_store_2d(&tmD, ebuf + buf * kEpiBufBytes, n0 + cp * 64, m0 + 32 * q);
-            bulk_commit_group();
-          }
-          buf ^= 1;
         }
         tc_fence_before();
         __syncwarp();
