@@ -137,10 +137,13 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def committed_traffic(wl, kept_tokens: int):
-    """Bytes per launch of the logits GEMM from the committed ncu capture, if the
-    kernel source is unchanged since; scaled to this workload's kept tokens x
-    vocabulary tiles (the reads also by d)."""
+def committed_traffic(wl, kept_tokens: int, kernel: str = "logits"):
+    """Bytes per launch of the logits or the dX GEMM from the committed ncu
+    capture, if the kernel source is unchanged since.  The logits GEMM's figure
+    is scaled to this workload's kept tokens x vocabulary tiles (the reads also
+    by d); the dX GEMM's (which reads the exponentials, W once per raster group
+    and the hidden rows, and writes dH) only to its kept tokens, at the captured
+    d and V (None otherwise)."""
     try:
         kv = {}
         with open(TRAFFIC_FILE) as f:
@@ -149,6 +152,12 @@ def committed_traffic(wl, kept_tokens: int):
                     k, v = ln.split("=", 1)
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_sha") != kernel_hash():
+            return None
+        if kernel == "dxhat":
+            if wl.d != int(kv["d"]) or wl.V != int(kv["V"]):
+                return None
+            return kept_tokens * float(kv["dxhat_dram_bytes_per_token"])
+        if kernel != "logits":
             return None
         w = float(kv["dram_write_bytes_per_token_per_vocab_tile"])
         r = float(kv["dram_read_bytes_per_token_per_vocab_tile"])
@@ -523,13 +532,16 @@ def run_ours(args, wl):
     else:
         names = sr.STAGE_NAMES
         # masked tokens are skipped: the logits and dX products run over the kept
-        # tokens; dW reduces over the final module's N rows (kept ones, then zeros)
-        gemm_stage_flops = {"logits": Gk, "dxhat": Gk, "dW": G / wl.K}
+        # tokens; dW reduces over the final module's kept tokens in whole blocks of
+        # 128 rows (the last one completed with zeros)
+        dw_rows = -(-(n_kept[-1] if n_kept[-1] > 0 else wl.N) // 128) * 128
+        gemm_stage_flops = {"logits": Gk, "dxhat": Gk,
+                            "dW": costmodel.gemm_flops(dw_rows, wl.V, wl.d)}
     dom = max(gemm_stage_flops, key=lambda s: stage_ms[names.index(s)])
     dom_ms = stage_ms[names.index(dom)]
     achieved = gemm_stage_flops[dom] / (dom_ms / 1e3) / 1e12
     peak, peak_name = tensor_peak(peaks, peak_src, ms / 1e3)
-    traffic = committed_traffic(wl, sum(n_kept)) if dom == "logits" and not onchip else None
+    traffic = None if onchip else committed_traffic(wl, sum(n_kept), dom)
     algo = costmodel.call_flops(wl.K, wl.N, wl.d, wl.V)
     kept = costmodel.kept_call_flops(n_kept, wl.d, wl.V)
     executed = sum(gemm_stage_flops.values())

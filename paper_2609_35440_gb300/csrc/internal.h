@@ -275,7 +275,6 @@ struct RowArgs {
   // every row goes through the gradient pass.
   float* row_fa;         // [M]
   float* row_fb;         // [M]
-  int32_t full_grad;     // 1: every row through the gradient pass (bias gradients)
   // Compaction of the kept tokens (null kept_local: every token keeps its row).
   // Kept tokens take rows [0, Mk) of the per-row buffers in token order, module
   // by module; each masked token zeroes one row of [Mk, M).

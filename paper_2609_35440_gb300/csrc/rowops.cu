@@ -409,10 +409,10 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
         // formed by the dX̂ epilogue (fb = 1 - p_y: the W_y term).  A final-module
         // row's target entry of P becomes -(1 - p_y) e^{lse} in the gradient
         // pass, so that tau/Nvalid e^{-lse} P is its whole G row (fb = 0).  The
-        // other rows (and every row when bias gradients are wanted) have the
-        // gradient pass turn P into G.
+        // gradient pass turns P into G for the other rows (and sums every row
+        // when bias gradients are wanted).
         const int kk = static_cast<int>(tok / a.N);
-        const bool factor = kept && !a.full_grad && !own_ref && l <= 60.f;
+        const bool factor = kept && !own_ref && l <= 60.f;
         a.row_fa[row] = factor ? expf(-l) : -1.f;
         a.row_fb[row] = (factor && kk < a.K - 1) ? -expm1f(-nll) : 0.f;
       }
@@ -561,11 +561,18 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
 
 // With the bias gradient: a CTA owns kGradRows rows of one module and 2048
 // columns (8 tiles), each thread one 8-column vector down those rows, so it
-// also sums dL/dz over its rows (fixed order, per row chunk).
+// also sums dL/dz over its rows (fixed order, per row chunk).  Rows whose
+// gradient is P times a per-row factor (row_fa >= 0) are summed the same way
+// but keep their exponentials in P: the dX̂ epilogue applies the factor to an
+// auxiliary row, and a final-module row gets its target entry and its x̂ row
+// scaled, as in the pass without bias gradients.
 __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
   __shared__ float cfac[kGradRows][8];     // exp(m_t - lse) / Nvalid per row and tile
   __shared__ float sgy[kGradRows];
   __shared__ int sy[kGradRows];
+  __shared__ unsigned char skeep[kGradRows];   // 1: P keeps the row's exponentials
+  __shared__ float sxs[kGradRows];             // final-module factor row: x̂ scale, else NaN
+  __shared__ unsigned short sty[kGradRows];    // its target entry (bf16 bits)
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int k = blockIdx.y / a.db_chunks;
   const int chunk = blockIdx.y - k * a.db_chunks;
@@ -599,8 +606,31 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
     }
     sgy[r] = kept ? expm1f(-a.nll[i]) * wr : 0.f;
     sy[r] = kept ? y : -1;
+    const bool factor = kept && a.row_fa != nullptr && a.row_fa[i] >= 0.f;
+    skeep[r] = factor ? 1 : 0;
+    const bool fin = factor && k == a.K - 1;
+    sxs[r] = fin ? tau * w * a.row_fa[i] : __int_as_float(0x7fc00000);
+    sty[r] = fin ? __bfloat16_as_ushort(__float2bfloat16(expm1f(-a.nll[i]) * expf(l))) : 0;
   }
   __syncthreads();
+  if (k == a.K - 1 && a.row_fa != nullptr) {
+    // x̂ rows of the final module's factor rows times tau/Nvalid e^{-lse}
+    // (G^T x̂ = P'^T (c x̂)); the CTAs of a row chunk share each row's vectors
+    const int nvd = a.d / 8;
+    const int v0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nvd / gridDim.x);
+    const int len = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nvd / gridDim.x) - v0;
+    for (int idx = threadIdx.x; len > 0 && idx < rows * len; idx += 256) {
+      const int r = idx / len;
+      const float c = sxs[r];
+      if (c != c) continue;
+      uint4* xr = reinterpret_cast<uint4*>(a.xhat + (row0 + r) * a.d) + v0 + (idx - r * len);
+      float f[8];
+      unpack8(*xr, f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) f[j] *= c;
+      *xr = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+    }
+  }
   const int vec = blockIdx.x * 256 + threadIdx.x;    // 8-column vector of this thread
   if (vec * 8 >= a.ldp) return;
   const int col0 = vec * 8;
@@ -633,8 +663,13 @@ __global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
         colsum[j] += g;
         f[j] = g * tau;
       }
-      P[r * stride] =
-          make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+      if (!skeep[r]) {
+        P[r * stride] =
+            make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+      } else if (static_cast<unsigned>(ycol) < 8u && sxs[r] == sxs[r]) {
+        // a final-module factor row: its target entry becomes (p_y - 1) e^{lse}
+        reinterpret_cast<unsigned short*>(P + r * stride)[ycol] = sty[r];
+      }
     }
   }
   if (!in_bounds(chunk < a.db_chunks && col0 + 8 <= a.ldp, a.flags)) return;

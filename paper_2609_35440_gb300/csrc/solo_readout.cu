@@ -353,7 +353,6 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   // stored exponentials allow it; with bias gradients every row takes the pass
   ra.row_fa = reinterpret_cast<float*>(ws + L.row_fa);
   ra.row_fb = reinterpret_cast<float*>(ws + L.row_fb);
-  ra.full_grad = dbias != nullptr ? 1 : 0;
 
   const uint64_t M = static_cast<uint64_t>(L.M);
   const uint64_t d = static_cast<uint64_t>(D.d);

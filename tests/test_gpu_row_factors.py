@@ -3,10 +3,10 @@
 The logits epilogue stores each tile's exponentials against the reference 0
 while the tile's maximum logit stays within +-64.  A row all of whose tiles
 did so (and whose log-sum-exp is at most 60) skips the gradient pass: the dX̂
-epilogue forms tau/Nvalid (e^{-lse} (P W) - (1 - p_y) W_y) itself.  The other
-rows, and the final module's (dW needs G), go through the gradient pass.
-These tests put auxiliary-module rows in each regime and compare every output
-with the fp64 oracle:
+epilogue forms tau/Nvalid (e^{-lse} (P W) - (1 - p_y) W_y) itself; a final-module
+row gets its target entry of P and its x̂ row scaled instead (dW = P'^T (c x̂)).
+The other rows go through the gradient pass.  These tests put auxiliary-module
+rows in each regime and compare every output with the fp64 oracle:
   - logits about 90 above the rest (a tile stored against its own maximum);
   - every logit of a row below -64;
   - many logits near 60, so that lse exceeds 60 while every tile stays in bound;
