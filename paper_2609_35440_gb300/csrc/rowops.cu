@@ -566,7 +566,7 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
 // but keep their exponentials in P: the dX̂ epilogue applies the factor to an
 // auxiliary row, and a final-module row gets its target entry and its x̂ row
 // scaled, as in the pass without bias gradients.
-__global__ void __launch_bounds__(256) grad_colsum_kernel(const RowArgs a) {
+__global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   __shared__ float cfac[kGradRows][8];     // exp(m_t - lse) / Nvalid per row and tile
   __shared__ float sgy[kGradRows];
   __shared__ int sy[kGradRows];
