@@ -284,6 +284,9 @@ struct RowArgs {
   int32_t* offsets;      // [K + 1] first compact row of each module; offsets[K] = Mk
   int32_t* orig_row;     // [M] compact row -> token row k * N + n
   int32_t* tgt_c;        // [M] target of a compact row
+  int32_t* grad_list;    // [M]: rows whose gradient pass takes the whole row
+  int32_t* grad_count;   // [1]: their number (zeroed by the kept-token scan)
+  int32_t grad_ctas;     // CTAs of the whole-row pass (a few per SM)
 };
 
 constexpr int kScanRows = 1024;  // tokens per block of the kept-token scan

@@ -113,7 +113,10 @@ __global__ void __launch_bounds__(1024) keep_offsets_kernel(const RowArgs a) {
     if (threadIdx.x == 1023) carry_s = carry + warp_sum[warp] + incl;
     __syncthreads();
   }
-  if (threadIdx.x == 0) a.offsets[a.K] = carry_s;
+  if (threadIdx.x == 0) {
+    a.offsets[a.K] = carry_s;
+    if (a.grad_count) *a.grad_count = 0;   // the gradient pass's row list starts empty
+  }
 }
 
 // ---- final RMSNorm: r_i = (mean_j h_ij^2 + eps)^-1/2, xhat = bf16(gamma h r) ------
@@ -486,76 +489,145 @@ __global__ void __launch_bounds__(256) module_mean_kernel(const RowArgs a) {
 // as expm1(-(lse - z_y)), from the lse - z_y that the log-sum-exp pass forms
 // without cancellation, so that p_y - 1 keeps its relative precision.
 
-// One row per CTA: contiguous 16-byte vectors across the row (the fastest
-// form; used when no bias gradient is needed).
-__global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
-  extern __shared__ float ctile[];
+// End of the rows past the kept ones that the dW product may read: its
+// reduction covers the final module's kept rows in whole 128-row blocks (its
+// N rows, rounded, when it keeps none), so those rows are zeroed.
+__device__ __forceinline__ int64_t dw_zero_end(const RowArgs& a, int64_t M) {
+  const int64_t fin0 = a.offsets[a.K - 1];
+  const int64_t kept = a.offsets[a.K] - fin0;
+  const int64_t span = kept > 0 ? kept : a.N;
+  return min(M, fin0 + (span + 127) / 128 * 128);
+}
+
+// The gradient pass without bias gradients, in two launches.
+// grad_classify_kernel: 32 rows per CTA.  One coalesced look at the rows decides
+// what each needs: the whole row (a kept row without a per-row factor: P
+// becomes G; a masked row without compaction), listed for grad_rows_kernel;
+// its target entry and x̂ row only (a final-module row with a factor: dW =
+// G^T x̂ = P'^T (c x̂)), done here by one warp; or nothing (an auxiliary row with
+// a factor: the dX̂ epilogue forms its gradient).  kGradZeroCtas more CTAs zero
+// the rows past the kept ones that dW reads, one row at a time each.
+constexpr int kGradRowsPerCta = 32;
+constexpr int kGradZeroCtas = 128;
+
+__global__ void __launch_bounds__(256) grad_classify_kernel(const RowArgs a) {
+  __shared__ int s_rows[kGradRowsPerCta];
+  __shared__ int s_count;
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  const int64_t row = blockIdx.x;
-  if (!in_bounds(row < M, a.flags)) return;
-  uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
-  const int nvec = a.ldp / 8;
-  // compacted: rows [0, Mk) are kept tokens; past them, the rows up to the
-  // final module's first row plus N rounded up to whole 128-row reduction
-  // blocks are zeroed (the dW product's reduction may read them), the rest is
-  // never read
+  const int64_t row_base = static_cast<int64_t>(blockIdx.x) * kGradRowsPerCta;
   const bool compact = a.kept_local != nullptr;
-  if (compact && row >= a.offsets[a.K - 1] + (a.N + 127) / 128 * 128) return;
-  if (a.row_fa != nullptr && (!compact || row < a.offsets[a.K]) && a.row_fa[row] >= 0.f) {
-    // rows whose gradient is P times a per-row factor keep their exponentials;
-    // a final-module row (dW = G^T xhat) gets its target entry and its xhat row
-    // scaled by that factor, tau/Nvalid e^{-lse}: G^T xhat = P'^T (c xhat)
-    const int64_t rk = row;
-    const bool final_row = compact ? rk >= a.offsets[a.K - 1] : rk >= static_cast<int64_t>(a.K - 1) * a.N;
-    if (!final_row) return;
+  const int64_t nchk = (M + kGradRowsPerCta - 1) / kGradRowsPerCta;
+  if (blockIdx.x >= nchk) {
+    if (!compact) return;
+    const int64_t zend = dw_zero_end(a, M);
+    const int nvec = a.ldp / 8;
+    for (int64_t row = a.offsets[a.K] + (blockIdx.x - nchk); row < zend; row += kGradZeroCtas) {
+      uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
+      for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
+    }
+    return;
+  }
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    const int64_t row = row_base + lane;
+    const int64_t mk = compact ? a.offsets[a.K] : M;
+    const int64_t fin0 = compact ? a.offsets[a.K - 1] : static_cast<int64_t>(a.K - 1) * a.N;
+    int kind = 0;                 // 1: the whole row, 2: target entry and x̂ row
+    if (row < mk) {
+      const bool factor = a.row_fa != nullptr && a.row_fa[row] >= 0.f;
+      kind = !factor ? 1 : row >= fin0 ? 2 : 0;
+    }
+    const unsigned below = (1u << lane) - 1u;
+    const unsigned whole = __ballot_sync(0xffffffffu, kind == 1);
+    int base = 0;
+    if (lane == 0 && whole != 0u) base = atomicAdd(a.grad_count, __popc(whole));
+    base = __shfl_sync(0xffffffffu, base, 0);
+    if (kind == 1 && in_bounds(base + __popc(whole & below) < M, a.flags))
+      a.grad_list[base + __popc(whole & below)] = static_cast<int32_t>(row);
+    const unsigned part = __ballot_sync(0xffffffffu, kind == 2);
+    if (kind == 2) s_rows[__popc(part & below)] = lane;
+    if (lane == 0) s_count = __popc(part);
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = warp; i < s_count; i += 8) {
+    const int64_t rk = row_base + s_rows[i];
     const int64_t tk = compact ? a.orig_row[rk] : rk;
     const int kf = static_cast<int>(tk / a.N);
     const int yf = compact ? a.tgt_c[rk] : a.targets[rk];
     const float tauf = a.tau ? a.tau[kf] : 1.f;
     const float c = tauf * a.inv_nvalid[kf] * a.row_fa[rk];
-    if (threadIdx.x == 0 && in_bounds(yf >= 0 && yf < a.V, a.flags))
+    if (lane == 0 && in_bounds(yf >= 0 && yf < a.V, a.flags))
       a.P[rk * a.ldp + yf] = __bfloat16_as_ushort(__float2bfloat16(expm1f(-a.nll[rk]) * expf(a.lse[rk])));
     uint4* xr = reinterpret_cast<uint4*>(a.xhat + rk * a.d);
-    for (int v = threadIdx.x; v < a.d / 8; v += 256) {
+    for (int v = lane; v < a.d / 8; v += 32) {
       float f[8];
       unpack8(xr[v], f);
 #pragma unroll
       for (int j = 0; j < 8; ++j) f[j] *= c;
       xr[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
     }
-    return;
   }
-  const int64_t tok = compact ? a.orig_row[row < a.offsets[a.K] ? row : 0] : row;
-  const int k = static_cast<int>(tok / a.N);
-  const int y = compact ? a.tgt_c[row < a.offsets[a.K] ? row : 0] : a.targets[row];
-  if (compact ? row >= a.offsets[a.K] : !token_kept(a, row, y)) {
-    for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
-    return;
-  }
-  const float tau = a.tau ? a.tau[k] : 1.f;
-  const float w = a.inv_nvalid[k] * tau;
-  const float l = a.lse[row];
-  for (int t = threadIdx.x; t < a.n_tiles_v; t += 256)
-    ctile[t] = expf(a.stats[static_cast<int64_t>(t) * M + row].x - l) * w;
-  const float gy = expm1f(-a.nll[row]) * w;    // p_y - 1 at full relative precision
-  __syncthreads();
-  for (int v = threadIdx.x; v < nvec; v += 256) {
-    const int v0 = v * 8;
-    if (v0 >= a.V) {
-      P[v] = make_uint4(0, 0, 0, 0);
-      continue;
+}
+
+// grad_rows_kernel: the listed rows, one per CTA at a time (a grid of a few CTAs
+// per SM walks the list), contiguous 16-byte vectors across the row.
+__global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
+  extern __shared__ float ctile[];
+  const int64_t M = static_cast<int64_t>(a.K) * a.N;
+  const bool compact = a.kept_local != nullptr;
+  const int nvec = a.ldp / 8;
+  const int count = *a.grad_count;
+  if (!in_bounds(count <= M, a.flags)) return;
+  for (int i = blockIdx.x; i < count; i += gridDim.x) {
+    const int64_t row = a.grad_list[i];
+    if (!in_bounds(row >= 0 && row < M, a.flags)) continue;    // uniform across the CTA
+    uint4* P = reinterpret_cast<uint4*>(a.P + row * a.ldp);
+    const int64_t tok = compact ? a.orig_row[row] : row;
+    const int k = static_cast<int>(tok / a.N);
+    const int y = compact ? a.tgt_c[row] : a.targets[row];
+    if (!compact && !token_kept(a, row, y)) {
+      for (int v = threadIdx.x; v < nvec; v += 256) P[v] = make_uint4(0, 0, 0, 0);
+      continue;                   // uniform across the CTA
     }
-    if (!in_bounds(v0 / kBN < a.n_tiles_v, a.flags)) continue;
-    const float c = ctile[v0 / kBN];
-    float f[8];
-    unpack8(P[v], f);
+    const float tau = a.tau ? a.tau[k] : 1.f;
+    const float w = a.inv_nvalid[k] * tau;
+    const float l = a.lse[row];
+    __syncthreads();              // the previous row's factors are no longer read
+    for (int t = threadIdx.x; t < a.n_tiles_v; t += 256)
+      ctile[t] = expf(a.stats[static_cast<int64_t>(t) * M + row].x - l) * w;
+    const float gy = expm1f(-a.nll[row]) * w;    // p_y - 1 at full relative precision
+    __syncthreads();
+    constexpr int kAhead = 4;                     // vectors in flight per thread
+    for (int vb = threadIdx.x; vb < nvec; vb += 256 * kAhead) {
+      uint4 in[kAhead];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      f[j] *= c;
-      if (v0 + j >= a.V) f[j] = 0.f;
-      if (v0 + j == y) f[j] = gy;
+      for (int u = 0; u < kAhead; ++u) {
+        const int v = vb + 256 * u;
+        if (v < nvec && v * 8 < a.V) in[u] = P[v];
+      }
+#pragma unroll
+      for (int u = 0; u < kAhead; ++u) {
+        const int v = vb + 256 * u;
+        if (v >= nvec) break;
+        const int v0 = v * 8;
+        if (v0 >= a.V) {
+          P[v] = make_uint4(0, 0, 0, 0);
+          continue;
+        }
+        if (!in_bounds(v0 / kBN < a.n_tiles_v, a.flags)) continue;
+        const float c = ctile[v0 / kBN];
+        float f[8];
+        unpack8(in[u], f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          f[j] *= c;
+          if (v0 + j >= a.V) f[j] = 0.f;
+          if (v0 + j == y) f[j] = gy;
+        }
+        P[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+      }
     }
-    P[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
   }
 }
 
@@ -577,15 +649,13 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   const int k = blockIdx.y / a.db_chunks;
   const int chunk = blockIdx.y - k * a.db_chunks;
   // compacted: module k's kept tokens are rows [offsets[k], offsets[k + 1]); the
-  // final module's chunks also zero the rows past Mk up to its first row plus N
-  // rounded up to whole 128-row reduction blocks, which the dW product may read
-  // (their contents are stale: written as zeros, never scaled)
+  // final module's chunks also zero the rows past Mk that the dW product may
+  // read (their contents are stale: written as zeros, never scaled)
   const bool compact = a.kept_local != nullptr;
   const int64_t mbase = compact ? a.offsets[k] : static_cast<int64_t>(k) * a.N;
   const int64_t mkept = compact ? a.offsets[k + 1] : mbase + a.N;
   const int64_t row0 = mbase + static_cast<int64_t>(chunk) * kGradRows;
-  const int64_t end = (compact && k < a.K - 1) ? mkept
-                      : compact ? min(M, mbase + (a.N + 127) / 128 * 128) : mbase + a.N;
+  const int64_t end = (compact && k < a.K - 1) ? mkept : compact ? dw_zero_end(a, M) : mbase + a.N;
   const int rows = row0 >= end ? 0 : static_cast<int>(end - row0 < kGradRows ? end - row0 : kGradRows);
   const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
   if (!in_bounds(k < a.K && row0 + rows <= M, a.flags)) return;
@@ -794,12 +864,16 @@ cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const size_t smem = static_cast<size_t>(a.n_tiles_v) * sizeof(float);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(grad_rows_kernel,
+    const cudaError_t e = cudaFuncSetAttribute(grad_rows_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  grad_rows_kernel<<<static_cast<unsigned>(M), 256, smem, s>>>(a);
+  const int64_t ctas = (M + kGradRowsPerCta - 1) / kGradRowsPerCta + kGradZeroCtas;
+  grad_classify_kernel<<<static_cast<unsigned>(ctas), 256, 0, s>>>(a);
+  cudaError_t e = launched();
+  if (e != cudaSuccess) return e;
+  grad_rows_kernel<<<static_cast<unsigned>(a.grad_ctas > 0 ? a.grad_ctas : 1), 256, smem, s>>>(a);
   return launched();
 }
 

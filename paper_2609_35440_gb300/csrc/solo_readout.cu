@@ -62,6 +62,7 @@ struct Layout {
   size_t stats = 0, xhat = 0, P = 0, dgp = 0;
   size_t usum = 0, sy = 0, part_tau = 0, db_part = 0, aux = 0, total = 0;
   size_t kept_local = 0, chunk_base = 0, offsets = 0, orig_row = 0, tgt_c = 0;
+  size_t grad_list = 0, grad_count = 0;
   size_t row_fa = 0, row_fb = 0;
   int aux_slots = 0;
   int nchunks = 0;
@@ -138,6 +139,9 @@ Layout make_layout(const solo_dims_t& d) {
   // per-row factors of the rows whose gradient the dX̂ epilogue forms
   L.row_fa = take(M * 4);
   L.row_fb = take(M * 4);
+  // rows whose gradient pass takes the whole row, and their count
+  L.grad_list = take(M * 4);
+  L.grad_count = take(4);
   L.total = off;
   return L;
 }
@@ -349,10 +353,14 @@ solo_status_t run(const solo_dims_t* dims, const solo_bf16_t* const* hidden,
   ra.offsets = reinterpret_cast<int32_t*>(ws + L.offsets);
   ra.orig_row = reinterpret_cast<int32_t*>(ws + L.orig_row);
   ra.tgt_c = reinterpret_cast<int32_t*>(ws + L.tgt_c);
-  // the auxiliary modules' gradients are formed in the dX̂ epilogue where the
-  // stored exponentials allow it; with bias gradients every row takes the pass
+  // gradients formed from the stored exponentials and per-row factors where
+  // they allow it: in the dX̂ epilogue (auxiliary rows), from a target entry and
+  // a scaled x̂ row (final-module rows)
   ra.row_fa = reinterpret_cast<float*>(ws + L.row_fa);
   ra.row_fb = reinterpret_cast<float*>(ws + L.row_fb);
+  ra.grad_list = reinterpret_cast<int32_t*>(ws + L.grad_list);
+  ra.grad_count = reinterpret_cast<int32_t*>(ws + L.grad_count);
+  ra.grad_ctas = 4 * sms;
 
   const uint64_t M = static_cast<uint64_t>(L.M);
   const uint64_t d = static_cast<uint64_t>(D.d);
