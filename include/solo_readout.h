@@ -452,7 +452,7 @@ uint64_t solo_readout_kernel_launches(void);
  *  - Problems whose solo_readout_workspace_bytes exceeds
  *    SOLO_STATIC_SCRATCH_BYTES are rejected with
  *    SOLO_ERR_EXCEEDS_STATIC_SCRATCH before anything is enqueued (roughly
- *    K*N*(2.047*V + 2*d + 56) bytes plus up to 32 MiB of partial tiles of the
+ *    K*N*(2.047*V + 2*d + 60) bytes plus up to 32 MiB of partial tiles of the
  *    backward products must fit; e.g. K=2, N=256, d=128, V=4096 uses about
  *    8.3 MiB).
  *  - The first call on a device looks up the device address of the scratch

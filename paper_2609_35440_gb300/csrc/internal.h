@@ -291,7 +291,7 @@ struct RowArgs {
 
 constexpr int kScanRows = 1024;  // tokens per block of the kept-token scan
 
-constexpr int kGradRows = 256;   // rows per CTA of the gradient pass
+constexpr int kGradRows = 128;   // rows per CTA of the bias-gradient pass
 
 // Kept-token scan (with a.kept_local): per-chunk counts and in-chunk ranks,
 // then the prefix over chunks and the modules' compact offsets.
