@@ -483,6 +483,8 @@ def run_ours(args, wl):
     for evl in step_evs:
         stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(n_stages)]
     stage_ms /= args.steps
+    # each call from its first stage's start to its last stage's end
+    call_ms = [evl[0].elapsed_time(evl[n_stages]) for evl in step_evs]
 
     ms = max_over_ranks(ms, dev)
     tokens_step = wl.M
@@ -572,6 +574,10 @@ def run_ours(args, wl):
         "executed_tflops": executed / step_s / 1e12,
         "executed_frac_of_peak": executed / step_s / 1e12 / peak,
         "stages_ms": {n: round(float(v), 4) for n, v in zip(names, stage_ms)},
+        # per call (first stage start to last stage end, CUDA events): the
+        # median and the minimum over the timed calls, beside the mean above
+        "call_ms": {"median": round(float(np.median(call_ms)), 4),
+                    "min": round(float(np.min(call_ms)), 4)},
         "roofline": {"bound": "tensor",
                      "kernel": ("auxiliary on-chip pass (tcgen05, cluster split of d)"
                                 if dom == "aux_onchip" else f"{dom} GEMM (tcgen05)"
@@ -641,6 +647,7 @@ def run_exit_bench(args, wl):
     for evl in evs:
         stage_ms += [evl[i].elapsed_time(evl[i + 1]) for i in range(sr.SOLO_EXIT_NUM_STAGES)]
     stage_ms /= args.steps
+    call_ms = [evl[0].elapsed_time(evl[sr.SOLO_EXIT_NUM_STAGES]) for evl in evs]
     flags = ex.flags(stream)
     value = job_throughput(wl.M, args.steps, 1, ms)
     # end to end: hidden states and targets from pinned host memory, losses and
@@ -690,6 +697,8 @@ def run_exit_bench(args, wl):
                    "parallelism": "replicas1",
                    "l2": l2_note(wl, False)},
         "stages_ms": {n: round(float(v), 4) for n, v in zip(sr.EXIT_STAGE_NAMES, stage_ms)},
+        "call_ms": {"median": round(float(np.median(call_ms)), 4),
+                    "min": round(float(np.min(call_ms)), 4)},
         "roofline": {"bound": "tensor", "kernel": "exit logits GEMM (tcgen05)",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None,
