@@ -646,8 +646,13 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   __shared__ float sxs[kGradRows];             // final-module factor row: x̂ scale, else NaN
   __shared__ unsigned short sty[kGradRows];    // its target entry (bf16 bits)
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
-  const int k = blockIdx.y / a.db_chunks;
-  const int chunk = blockIdx.y - k * a.db_chunks;
+  // one-dimensional grid, the 2048-column slice fastest (the CTAs running
+  // together read whole rows): blockIdx.x = (module, row chunk) * slices + slice
+  const int nslice = (a.ldp / 8 + 255) / 256;
+  const int slice = static_cast<int>(blockIdx.x % static_cast<unsigned>(nslice));
+  const int unit = static_cast<int>(blockIdx.x / static_cast<unsigned>(nslice));
+  const int k = unit / a.db_chunks;
+  const int chunk = unit - k * a.db_chunks;
   // compacted: module k's kept tokens are rows [offsets[k], offsets[k + 1]); the
   // final module's chunks also zero the rows past Mk that the dW product may
   // read (their contents are stale: written as zeros, never scaled)
@@ -657,7 +662,7 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   const int64_t row0 = mbase + static_cast<int64_t>(chunk) * kGradRows;
   const int64_t end = (compact && k < a.K - 1) ? mkept : compact ? dw_zero_end(a, M) : mbase + a.N;
   const int rows = row0 >= end ? 0 : static_cast<int>(end - row0 < kGradRows ? end - row0 : kGradRows);
-  const int t0 = blockIdx.x * 8;                 // first 256-column tile of this CTA
+  const int t0 = slice * 8;                      // first 256-column tile of this CTA
   if (!in_bounds(k < a.K && row0 + rows <= M, a.flags)) return;
   const float w = a.inv_nvalid[k];
   const float tau = a.tau ? a.tau[k] : 1.f;
@@ -687,8 +692,8 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
     // x̂ rows of the final module's factor rows times tau/Nvalid e^{-lse}
     // (G^T x̂ = P'^T (c x̂)); the CTAs of a row chunk share each row's vectors
     const int nvd = a.d / 8;
-    const int v0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nvd / gridDim.x);
-    const int len = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nvd / gridDim.x) - v0;
+    const int v0 = static_cast<int>(static_cast<int64_t>(slice) * nvd / nslice);
+    const int len = static_cast<int>(static_cast<int64_t>(slice + 1) * nvd / nslice) - v0;
     for (int idx = threadIdx.x; len > 0 && idx < rows * len; idx += 256) {
       const int r = idx / len;
       const float c = sxs[r];
@@ -701,7 +706,7 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
       *xr = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
     }
   }
-  const int vec = blockIdx.x * 256 + threadIdx.x;    // 8-column vector of this thread
+  const int vec = slice * 256 + threadIdx.x;         // 8-column vector of this thread
   if (vec * 8 >= a.ldp) return;
   const int col0 = vec * 8;
   const int tt = threadIdx.x >> 5;                    // 32 vectors = one 256-column tile
@@ -854,8 +859,8 @@ cudaError_t launch_exit_lse(const RowArgs& a, cudaStream_t s) {
 
 cudaError_t launch_grad(const RowArgs& a, cudaStream_t s) {
   if (a.dbias) {
-    const dim3 grid((a.ldp / 8 + 255) / 256, a.K * a.db_chunks);
-    grad_colsum_kernel<<<grid, 256, 0, s>>>(a);
+    const int64_t ctas = static_cast<int64_t>(a.K) * a.db_chunks * ((a.ldp / 8 + 255) / 256);
+    grad_colsum_kernel<<<static_cast<unsigned>(ctas), 256, 0, s>>>(a);
     cudaError_t e = launched();
     if (e != cudaSuccess) return e;
     dbias_reduce_kernel<<<dim3((a.V + 255) / 256, a.K), 256, 0, s>>>(a);
