@@ -207,7 +207,7 @@ __device__ __forceinline__ uint32_t xhat_bf16x2(float gh0, float gh1, F2 r) {
 // VPL > 0: the row is held in registers (VPL 16-byte vectors per lane, d <=
 // 256 * VPL), so h is read from memory once.  VPL == 0: any d, h re-read.
 template <int VPL>
-__global__ void __launch_bounds__(256) rmsnorm_fwd_kernel(const RowArgs a) {
+__global__ void __launch_bounds__(256, 4) rmsnorm_fwd_kernel(const RowArgs a) {
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   const int lane = threadIdx.x & 31;
   const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
