@@ -181,6 +181,7 @@ class ClockSampler:
     def __init__(self, index: int):
         self.index = 0 if index is None else index
         self.proc = None
+        self.window = None          # (first, last) sample indices of the timed region
         self.lines = []
 
     def __enter__(self):
@@ -212,10 +213,32 @@ class ClockSampler:
                 self.proc.kill()
             self.thread.join(timeout=2)
 
+    def mark_start(self):
+        """Call right before the timed region is enqueued."""
+        self.window = (len(self.lines), None)
+
+    def mark_end(self):
+        """Call once the timed region has completed on the device.  A region
+        shorter than the sampling period waits (at most a second) for the first
+        sample after its start."""
+        if self.window is None:
+            return
+        t0 = time.time()
+        while (len(self.lines) <= self.window[0] and self.proc is not None
+               and self.proc.poll() is None and time.time() - t0 < 1.0):
+            time.sleep(0.005)
+        self.window = (self.window[0], len(self.lines))
+
     def summary(self):
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        lines = self.lines
+        if self.window is not None and self.window[1] is not None:
+            # the samples taken while the timed calls ran; a region shorter than
+            # the sampling period keeps the first sample after its start
+            lo, hi = self.window
+            lines = self.lines[lo:max(hi, lo + 1)]
+        for ln in lines:
             parts = [x.strip() for x in ln.split(",")]
             if len(parts) < 8:
                 continue
@@ -224,12 +247,18 @@ class ClockSampler:
                 mx.append(float(parts[1]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(parts[2]))
+            except ValueError:
+                pass
             for nm, v in zip(names, parts[4:8]):
                 if v.lower().startswith("active"):
                     reasons.add(nm)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "sm_mhz_min": min(sm),
+                "power_w": statistics.median(pw) if pw else None,
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
@@ -475,12 +504,14 @@ def run_ours(args, wl):
     t1 = torch.cuda.Event(enable_timing=True)
     barrier()
     launches0 = sr.solo_readout_kernel_launches()
+    clk.mark_start()
     t0.record(stream)
     for i in range(args.steps):
         ro(hidden, gamma, W, targets, stream=stream, events=step_evs[i], **heads)
     t1.record(stream)
     launches = sr.solo_readout_kernel_launches() - launches0
     barrier()
+    clk.mark_end()
     clk.__exit__(None, None, None)
     flags = ro.flags(stream)
     ms = t0.elapsed_time(t1)
@@ -640,12 +671,14 @@ def run_exit_bench(args, wl):
     t1 = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize(dev)
     launches0 = sr.solo_readout_kernel_launches()
+    clk.mark_start()
     t0.record(stream)
     for i in range(args.steps):
         ex(hidden, gamma, W, targets, stream=stream, events=evs[i])
     t1.record(stream)
     launches = sr.solo_readout_kernel_launches() - launches0
     torch.cuda.synchronize(dev)
+    clk.mark_end()
     clk.__exit__(None, None, None)
     ms = t0.elapsed_time(t1)
     stage_ms = np.zeros(sr.SOLO_EXIT_NUM_STAGES)
@@ -756,12 +789,14 @@ def run_private_bench(args, wl):
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     launches0 = sr.solo_readout_kernel_launches()
+    clk.mark_start()
     t0.record(stream)
     for _ in range(args.steps):
         call()
     t1.record(stream)
     launches = sr.solo_readout_kernel_launches() - launches0
     torch.cuda.synchronize(dev)
+    clk.mark_end()
     clk.__exit__(None, None, None)
     ms = t0.elapsed_time(t1)
     peaks, peak_src = load_peaks()
