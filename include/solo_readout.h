@@ -80,7 +80,11 @@ enum {
   SOLO_STAGE_RMSNORM = 0,   /* r_i and xhat = bf16(gamma * h * r)           */
   SOLO_STAGE_LOGITS = 1,    /* tensor-core X W^T, per-tile max/sum, exps    */
   SOLO_STAGE_LSE = 2,       /* logsumexp, token loss, module means          */
-  SOLO_STAGE_GRAD = 3,      /* dL/dz = (softmax - onehot) / Nvalid, bf16    */
+  SOLO_STAGE_GRAD = 3,      /* dL/dz = tau (softmax - onehot) / Nvalid: the
+                               per-row factors of most rows applied in place
+                               (final module: target entry, scaled xhat),
+                               bf16 G written for the rest (with bias
+                               gradients: every row summed into db)          */
   SOLO_STAGE_DXHAT = 4,     /* tensor-core dXhat = G W; its epilogue takes
                                dH through the RMSNorm Jacobian and forms the
                                dgamma partial sums                           */
@@ -103,7 +107,8 @@ typedef struct {
 /*
  * Bytes of device workspace one call with these dims needs (host-only; no
  * CUDA call).  The workspace holds the normalised inputs, the bf16
- * exponentials/gradient of the logits ([K*N, V]), per-token statistics,
+ * exponentials/gradient of the logits ([K*N, V], one row per kept token),
+ * per-token statistics and factors,
  * at most 32 MiB of fp32 partial tiles of the backward products and the flag
  * word.  Returns SOLO_ERR_INVALID_ARG for NULL pointers or dims out of range,
  * SOLO_ERR_UNSUPPORTED_SHAPE when d % 8 != 0 or V > 2^23.
