@@ -99,10 +99,10 @@ def test_heads_reference_choices(sr, neg_tau, bias_std):
 
 def test_without_heads_is_the_plain_call_bitwise(sr):
     """tau = 1 and b = 0 give the plain call's results bit for bit.  With the
-    bias gradient requested every row's G goes through the gradient pass (the
-    plain call forms most rows' gradient from the stored exponentials times a
-    per-row factor), so the gradients then agree within the parity tolerances
-    and the losses still bit for bit."""
+    bias gradient requested the bias-gradient pass sums every row's G and
+    rewrites the rows without per-row factors in its own order of rounding
+    (tau applied last), so the gradients then agree within the parity
+    tolerances and the losses still bit for bit."""
     wl = SMALL[1]
     inp = synth.generate(wl)
     plain = parity.run_gpu(wl, inp)
