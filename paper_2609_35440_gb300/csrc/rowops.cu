@@ -314,6 +314,9 @@ __global__ void __launch_bounds__(256, 4) rmsnorm_fwd_kernel(const RowArgs a) {
 
 enum LseKind { kLseTrain = 0, kLseExit = 1, kLseHeads = 2 };
 
+// tiles whose statistics one thread loads together (independent loads in flight)
+constexpr int kLseBatch = 16;
+
 // kLseExit: also the first argmax over the vocabulary and its log-probability;
 // targets may be absent (decoding only).  kLseHeads: also the temperature's
 // gradient term E_p[s] - s_y of every kept token (s: logits before the
@@ -345,18 +348,18 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       const int y0 = tgt ? tgt[row] : a.ignore_index;
       if (compact || token_kept(a, row, y0)) ys = kHeads ? a.sy[row] : a.zy[row];
     }
-    for (int t0 = 0; t0 < a.n_tiles_v; t0 += 8) {
-      float2 st[8];
-      float uu[8];
+    for (int t0 = 0; t0 < a.n_tiles_v; t0 += kLseBatch) {
+      float2 st[kLseBatch];
+      float uu[kLseBatch];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {       // independent loads, issued together
+      for (int u = 0; u < kLseBatch; ++u) {       // independent loads, issued together
         const bool in = t0 + u < a.n_tiles_v;
         st[u] = in ? a.stats[static_cast<int64_t>(t0 + u) * M + row] : make_float2(-INFINITY, 0.f);
         if constexpr (!kExit) uu[u] = in ? a.usum[static_cast<int64_t>(t0 + u) * M + row] : 0.f;
       }
       float cm = mx;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kLseBatch; ++u) {
         if (kExit && st[u].x > cm) best_tile = t0 + u;   // strict: the first tile with the max
         cm = fmaxf(cm, st[u].x);
         if (!kExit && t0 + u < a.n_tiles_v && st[u].x != 0.f) own_ref = true;
@@ -365,7 +368,7 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
       s *= rescale;
       if constexpr (!kExit) us *= rescale;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kLseBatch; ++u) {
         const float f = expf(st[u].x - cm);
         s += st[u].y * f;
         if constexpr (!kExit) {
