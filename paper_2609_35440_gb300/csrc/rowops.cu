@@ -389,9 +389,15 @@ __global__ void __launch_bounds__(256) lse_kernel(const RowArgs a) {
     } else {
       if (y >= 0 && y < a.V) {
         // the tile sums leave the target's term out: lse - z_y without
-        // cancellation (mx >= z_y, equal when the target holds the maximum)
+        // cancellation.  u = sum over v != y of e^{z_v - z_y} (inf when it
+        // overflows).  While u <= 1 (p_y >= 1/2) log1p(u) keeps 1 - p_y's
+        // relative precision, whatever the reference mx is: it is 0 for the
+        // tiles whose logits stay within +-64, so a confident target may lie
+        // below it.  Otherwise lse - z_y >= ln 2 and the second form does not
+        // cancel.
         const float zt = a.zy[row];
-        nll = zt >= mx ? log1pf(s * expf(mx - zt)) : (mx - zt) + logf(s + expf(zt - mx));
+        const float u = s > 0.f ? s * expf(mx - zt) : 0.f;
+        nll = (zt >= mx || u <= 1.f) ? log1pf(u) : (mx - zt) + logf(s + expf(zt - mx));
         l = zt + nll;
         a.nll[row] = nll;
       }

@@ -59,6 +59,24 @@ def test_ragged_shapes(wl):
     parity.compare_full(wl, gpu, ref)
 
 
+# Vocabularies narrower than one 64-column TMA box and than the 16-byte row of
+# the exponential buffer: the loads past V read zeros, the stores past V are
+# dropped, and with V = 1 every loss and gradient is exactly zero.
+TINY_V = [Workload(f"k2_n50_d64_v{V}", K=2, N=50, d=64, V=V, seed=60 + V, mask_frac=0.1)
+          for V in (1, 3, 8, 13)]
+
+
+@pytest.mark.parametrize("wl", TINY_V, ids=lambda w: w.name)
+def test_tiny_vocabulary(wl):
+    _, gpu, ref = _case(wl)
+    assert gpu["flags"] == 0
+    parity.compare_full(wl, gpu, ref)
+    if wl.V == 1:
+        assert not np.any(gpu["loss_tok"]) and not np.any(gpu["dW"])
+        for k in range(wl.K):
+            assert not np.any(gpu["dhidden"][k])
+
+
 # Every GEMM runs several work units per CTA pair here (76 pairs on GB300), so
 # the second TMEM accumulator, its phase flips and raster groups beyond the
 # first are compared element by element:
