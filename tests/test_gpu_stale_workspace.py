@@ -8,8 +8,8 @@ multiple of the 128-row reduction blocks, so the dW product's last block
 reaches past the final module's kept rows: those rows must be zeros written by
 the gradient pass, not what an earlier call left there.  Checked for the plain
 call (rows whose gradient is P times a per-row factor), for the heads' call
-with the bias gradient (every row through the gradient pass), and for a second
-call on the same workspace with a different mask.
+with the bias gradient, for a second call on the same workspace with a
+different mask, and for the on-chip call and the exit readout.
 """
 import numpy as np
 import pytest
@@ -117,3 +117,33 @@ def test_second_call_with_fewer_kept_tokens(sr):
     gpu = _call(sr, WL, inp, ro)
     assert gpu["flags"] == 0
     parity.compare_full(WL, gpu, _oracle(WL, inp))
+
+
+def test_onchip_call_on_a_poisoned_workspace(sr):
+    inp = synth.generate(WL)
+    ro = sr.Readout(WL.K, WL.N, WL.d, WL.V, eps=WL.eps, onchip=True)
+    _poison(ro)
+    gpu = _call(sr, WL, inp, ro)
+    assert gpu["flags"] == 0
+    parity.compare_full(WL, gpu, _oracle(WL, inp))
+
+
+def test_exit_readout_on_a_poisoned_workspace(sr):
+    import torch
+    from tests.test_gpu_exit import _compare
+    inp = synth.generate(WL)
+    ex = sr.ExitReadout(WL.K, WL.N, WL.d, WL.V, eps=WL.eps)
+    ex.workspace.fill_(0xFF)
+    for t in (ex.loss_tok, ex.loss_mean, ex.top1, ex.top1_logprob):
+        t.view(torch.uint8).fill_(0xFF)
+    hidden = [parity.to_device_bf16(inp.hidden[k]) for k in range(WL.K)]
+    gamma, W = parity.to_device_bf16(inp.gamma), parity.to_device_bf16(inp.W)
+    tg = torch.from_numpy(np.ascontiguousarray(inp.targets, dtype=np.int32)).cuda()
+    ex(hidden, gamma, W, tg)
+    torch.cuda.synchronize()
+    gpu = dict(top1=ex.top1.cpu().numpy(), top1_logprob=ex.top1_logprob.double().cpu().numpy(),
+               loss_tok=ex.loss_tok.double().cpu().numpy(),
+               loss_mean=ex.loss_mean.double().cpu().numpy(), flags=ex.flags())
+    assert gpu["flags"] == 0
+    _compare(WL, inp, gpu)
+    np.testing.assert_allclose(gpu["loss_mean"], _oracle(WL, inp)["loss_mean"], rtol=1e-5, atol=0)
