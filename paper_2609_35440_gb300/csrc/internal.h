@@ -267,12 +267,13 @@ struct RowArgs {
   float* dtau;           // [K] or null
   float* dbias;          // [K, V] or null
   float* db_part;        // [K, db_chunks, ldp]
-  int32_t db_chunks;     // row chunks per module of the gradient pass
-  // Rows whose gradient the dX̂ epilogue forms (the log-sum-exp pass decides):
-  // row_fa = e^{-lse} and row_fb = 1 - p_y for them, row_fa = -1 for the rows
-  // the gradient pass turns into G (the final module's, whose dW needs G, and
-  // rows with a tile stored against its own maximum or lse above 60).  Null:
-  // every row goes through the gradient pass.
+  int32_t db_chunks;     // row chunks per module of the bias-gradient pass
+  // Rows whose gradient is the stored exponentials times per-row factors (the
+  // log-sum-exp pass decides): row_fa = e^{-lse}, and row_fb = 1 - p_y for an
+  // auxiliary row (the dX̂ epilogue's W_y term) or 0 for a final-module row
+  // (its target entry and x̂ row are rewritten instead).  row_fa = -1 for the
+  // rows the gradient pass turns into G (a tile stored against its own
+  // maximum, or lse above 60).  Null: every row goes through the gradient pass.
   float* row_fa;         // [M]
   float* row_fb;         // [M]
   // Compaction of the kept tokens (null kept_local: every token keeps its row).
