@@ -586,8 +586,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          if (even) mbar_arrive(&tempty[acc]);
-          else mbar_arrive_remote(tempty_even + acc * 8);
+          if (even) mbar_arrive_relaxed(&tempty[acc]);
+          else mbar_arrive_remote_relaxed(tempty_even + acc * 8);
         }
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
           args.stats[static_cast<size_t>(nb) * args.M + row] = make_float2(mx, ssum);
@@ -759,8 +759,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          if (even) mbar_arrive(&tempty[acc]);
-          else mbar_arrive_remote(tempty_even + acc * 8);
+          if (even) mbar_arrive_relaxed(&tempty[acc]);
+          else mbar_arrive_remote_relaxed(tempty_even + acc * 8);
         }
         const float ssum = sacc.x + sacc.y;
         if (row_ok && in_bounds(nb < args.n_blocks, args.flags)) {
@@ -786,8 +786,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          if (even) mbar_arrive(&tempty[acc]);
-          else mbar_arrive_remote(tempty_even + acc * 8);
+          if (even) mbar_arrive_relaxed(&tempty[acc]);
+          else mbar_arrive_remote_relaxed(tempty_even + acc * 8);
         }
       } else {
         for (int c = 0; c < kBN / 32; ++c) {
@@ -824,8 +824,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          if (even) mbar_arrive(&tempty[acc]);
-          else mbar_arrive_remote(tempty_even + acc * 8);
+          if (even) mbar_arrive_relaxed(&tempty[acc]);
+          else mbar_arrive_remote_relaxed(tempty_even + acc * 8);
         }
       }
     }
