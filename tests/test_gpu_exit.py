@@ -84,6 +84,20 @@ SMALL = [workloads.SMOKE,
                   heavy_frac=0.01, row_scale=True, mask_frac=0.05)]
 
 
+TINY_V = [Workload(f"exit_k2_n50_d64_v{V}", K=2, N=50, d=64, V=V, seed=70 + V, mask_frac=0.1)
+          for V in (2, 3, 13)]
+
+
+@pytest.mark.parametrize("wl", TINY_V, ids=lambda w: w.name)
+def test_exit_readout_tiny_vocabulary(sr, wl):
+    """Vocabularies narrower than one 32-column chunk of the epilogue."""
+    inp = synth.generate(wl)
+    gpu = _gpu_exit(sr, wl, inp)
+    assert gpu["flags"] == 0
+    _compare(wl, inp, gpu)
+    assert np.all((gpu["top1"] >= 0) & (gpu["top1"] < wl.V))
+
+
 @pytest.mark.parametrize("wl", SMALL, ids=lambda w: w.name)
 def test_exit_readout_small(sr, wl):
     inp = synth.generate(wl)

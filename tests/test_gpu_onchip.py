@@ -55,6 +55,18 @@ SHAPES = [
 ]
 
 
+TINY_V = [Workload(f"onchip_k2_n50_d64_v{V}", K=2, N=50, d=64, V=V, seed=80 + V, mask_frac=0.1)
+          for V in (1, 3)]
+
+
+@pytest.mark.parametrize("wl", TINY_V, ids=lambda w: w.name)
+def test_onchip_tiny_vocabulary(wl):
+    """One vocabulary tile, almost all of it past V: masked out of every sum."""
+    _, gpu, ref = _case(wl)
+    assert gpu["flags"] == 0
+    parity.compare_full(wl, gpu, ref)
+
+
 @pytest.mark.parametrize("wl", SHAPES, ids=lambda w: w.name)
 def test_onchip_full_parity(wl):
     _, gpu, ref = _case(wl)
