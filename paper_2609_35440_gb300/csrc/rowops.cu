@@ -725,6 +725,7 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   uint4* P = reinterpret_cast<uint4*>(a.P + row0 * a.ldp) + vec;
   const int64_t stride = a.ldp / 8;
   constexpr int kAhead = 8;                           // rows in flight per thread
+  const bool vfull = col0 + 8 <= a.V;                 // every column of the vector in V
   for (int r0 = 0; r0 < rows; r0 += kAhead) {
     uint4 in[kAhead];
 #pragma unroll
@@ -734,22 +735,31 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
     for (int u = 0; u < kAhead; ++u) {
       const int r = r0 + u;
       if (r >= rows) break;
-      const float c = cfac[r][tt];
-      const bool live = sy[r] >= 0;
-      const int ycol = sy[r] - col0;
-      float f[8];
-      unpack8(in[u], f);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float g = live ? f[j] * c : 0.f;
-        if (j == ycol) g = sgy[r];
-        if (col0 + j >= a.V) g = 0.f;
-        colsum[j] += g;
-        f[j] = g * tau;
+      const int yr = sy[r];
+      if (yr < 0) {                 // a masked or zero row (warp-uniform): G = 0
+        P[r * stride] = make_uint4(0, 0, 0, 0);
+        continue;
       }
+      const float c = cfac[r][tt];
+      const int ycol = yr - col0;
+      float g[8];
+      unpack8(in[u], g);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) g[j] *= c;
+      if (static_cast<unsigned>(ycol) < 8u) {      // the thread holding the target
+        const float gy = sgy[r];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) g[j] = j == ycol ? gy : g[j];
+      }
+      if (!vfull) {                 // the vector that crosses V
+#pragma unroll
+        for (int j = 0; j < 8; ++j) g[j] = col0 + j < a.V ? g[j] : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) colsum[j] += g[j];
       if (!skeep[r]) {
-        P[r * stride] =
-            make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
+        P[r * stride] = make_uint4(pack2(g[0] * tau, g[1] * tau), pack2(g[2] * tau, g[3] * tau),
+                                   pack2(g[4] * tau, g[5] * tau), pack2(g[6] * tau, g[7] * tau));
       } else if (static_cast<unsigned>(ycol) < 8u && sxs[r] == sxs[r]) {
         // a final-module factor row: its target entry becomes (p_y - 1) e^{lse}
         reinterpret_cast<unsigned short*>(P + r * stride)[ycol] = sty[r];
