@@ -629,10 +629,15 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
         float f[8];
         unpack8(in[u], f);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          f[j] *= c;
-          if (v0 + j >= a.V) f[j] = 0.f;
-          if (v0 + j == y) f[j] = gy;
+        for (int j = 0; j < 8; ++j) f[j] *= c;
+        if (v0 + 8 > a.V) {          // the vector that crosses V
+#pragma unroll
+          for (int j = 0; j < 8; ++j) f[j] = v0 + j < a.V ? f[j] : 0.f;
+        }
+        const int ycol = y - v0;
+        if (static_cast<unsigned>(ycol) < 8u) {   // the vector holding the target
+#pragma unroll
+          for (int j = 0; j < 8; ++j) f[j] = j == ycol ? gy : f[j];
         }
         P[v] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
       }
