@@ -6,8 +6,9 @@ tensor memory reused before its epilogue finished reading it, a stage of the
 operand ring refilled before its MMAs completed, or rows of the gradient
 pass's list processed twice or not at all.  The call runs back to back many
 times (at full size, so that every persistent GEMM runs many work units per
-CTA pair, in the plain and in the heads' mode) and each output is compared on
-the device with the first call's.
+CTA pair, in the plain and the heads' mode and the on-chip call, whose
+clusters exchange partial logits through distributed shared memory) and each
+output is compared on the device with the first call's.
 """
 import numpy as np
 import pytest
@@ -37,20 +38,21 @@ def _outputs(ro, heads):
     return [t.clone() for t in outs]
 
 
-@pytest.mark.parametrize("heads", [False, True], ids=["plain", "heads"])
-def test_back_to_back_calls_are_bitwise_equal(sr, heads):
+@pytest.mark.parametrize("mode", ["plain", "heads", "onchip"])
+def test_back_to_back_calls_are_bitwise_equal(sr, mode):
     import torch
     wl = workloads.W1P3B
     inp = synth.generate(wl)
     hidden = [parity.to_device_bf16(inp.hidden[k]) for k in range(wl.K)]
     gamma, W = parity.to_device_bf16(inp.gamma), parity.to_device_bf16(inp.W)
     tg = torch.from_numpy(np.ascontiguousarray(inp.targets, dtype=np.int32)).cuda()
+    heads = mode == "heads"
     kw = {}
     if heads:
         tau, bias = synth.gen_heads(wl)
         kw = dict(tau=torch.from_numpy(tau).cuda(), bias=torch.from_numpy(bias).cuda(),
                   head_grads=True)
-    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps)
+    ro = sr.Readout(wl.K, wl.N, wl.d, wl.V, eps=wl.eps, onchip=mode == "onchip")
     ro(hidden, gamma, W, tg, **kw)
     first = _outputs(ro, heads)
     mismatches = torch.zeros(len(first), dtype=torch.int64, device="cuda")
