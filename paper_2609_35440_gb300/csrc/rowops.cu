@@ -654,11 +654,11 @@ __global__ void __launch_bounds__(256) grad_rows_kernel(const RowArgs a) {
 // scaled, as in the pass without bias gradients.
 __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
   __shared__ float cfac[kGradRows][8];     // exp(m_t - lse) / Nvalid per row and tile
-  __shared__ float sgy[kGradRows];
-  __shared__ int sy[kGradRows];
-  __shared__ unsigned char skeep[kGradRows];   // 1: P keeps the row's exponentials
-  __shared__ float sxs[kGradRows];             // final-module factor row: x̂ scale, else NaN
-  __shared__ unsigned short sty[kGradRows];    // its target entry (bf16 bits)
+  // per row, read together: the target (-1: masked or zero row), (p_y - 1) /
+  // Nvalid, the x̂ scale of a final-module factor row (else NaN), and 1 when P
+  // keeps the row's exponentials
+  __shared__ float4 srow[kGradRows];
+  __shared__ unsigned short sty[kGradRows];    // a final-module factor row's target entry
   const int64_t M = static_cast<int64_t>(a.K) * a.N;
   // one-dimensional grid, the 2048-column slice fastest (the CTAs running
   // together read whole rows): blockIdx.x = (module, row chunk) * slices + slice
@@ -693,12 +693,11 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
       cfac[r][tt] = (wr != 0.f && t < a.n_tiles_v)
                         ? expf(a.stats[static_cast<int64_t>(t) * M + i].x - l) * wr : 0.f;
     }
-    sgy[r] = kept ? expm1f(-a.nll[i]) * wr : 0.f;
-    sy[r] = kept ? y : -1;
     const bool factor = kept && a.row_fa != nullptr && a.row_fa[i] >= 0.f;
-    skeep[r] = factor ? 1 : 0;
     const bool fin = factor && k == a.K - 1;
-    sxs[r] = fin ? tau * w * a.row_fa[i] : __int_as_float(0x7fc00000);
+    srow[r] = make_float4(__int_as_float(kept ? y : -1), kept ? expm1f(-a.nll[i]) * wr : 0.f,
+                          fin ? tau * w * a.row_fa[i] : __int_as_float(0x7fc00000),
+                          __int_as_float(factor ? 1 : 0));
     sty[r] = fin ? __bfloat16_as_ushort(__float2bfloat16(expm1f(-a.nll[i]) * expf(l))) : 0;
   }
   __syncthreads();
@@ -710,7 +709,7 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
     const int len = static_cast<int>(static_cast<int64_t>(slice + 1) * nvd / nslice) - v0;
     for (int idx = threadIdx.x; len > 0 && idx < rows * len; idx += 256) {
       const int r = idx / len;
-      const float c = sxs[r];
+      const float c = srow[r].z;
       if (c != c) continue;
       uint4* xr = reinterpret_cast<uint4*>(a.xhat + (row0 + r) * a.d) + v0 + (idx - r * len);
       float f[8];
@@ -740,7 +739,8 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
     for (int u = 0; u < kAhead; ++u) {
       const int r = r0 + u;
       if (r >= rows) break;
-      const int yr = sy[r];
+      const float4 rd = srow[r];
+      const int yr = __float_as_int(rd.x);
       if (yr < 0) {                 // a masked or zero row (warp-uniform): G = 0
         P[r * stride] = make_uint4(0, 0, 0, 0);
         continue;
@@ -752,7 +752,7 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
 #pragma unroll
       for (int j = 0; j < 8; ++j) g[j] *= c;
       if (static_cast<unsigned>(ycol) < 8u) {      // the thread holding the target
-        const float gy = sgy[r];
+        const float gy = rd.y;
 #pragma unroll
         for (int j = 0; j < 8; ++j) g[j] = j == ycol ? gy : g[j];
       }
@@ -762,10 +762,10 @@ __global__ void __launch_bounds__(256, 4) grad_colsum_kernel(const RowArgs a) {
       }
 #pragma unroll
       for (int j = 0; j < 8; ++j) colsum[j] += g[j];
-      if (!skeep[r]) {
+      if (__float_as_int(rd.w) == 0) {
         P[r * stride] = make_uint4(pack2(g[0] * tau, g[1] * tau), pack2(g[2] * tau, g[3] * tau),
                                    pack2(g[4] * tau, g[5] * tau), pack2(g[6] * tau, g[7] * tau));
-      } else if (static_cast<unsigned>(ycol) < 8u && sxs[r] == sxs[r]) {
+      } else if (static_cast<unsigned>(ycol) < 8u && rd.z == rd.z) {
         // a final-module factor row: its target entry becomes (p_y - 1) e^{lse}
         reinterpret_cast<unsigned short*>(P + r * stride)[ycol] = sty[r];
       }
